@@ -1,0 +1,20 @@
+"""Plain float64 CPU oracle for the sparse-prefill evidence probe.
+
+TEST INFRASTRUCTURE ONLY. Nothing in the product path imports this package:
+only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` may call it. It shares no code with
+the CUDA path; the only common module is the seeded input generator.
+
+Every function here follows the paper's statement of the probe:
+  * masked softmax attention restricted to retained blocks (Sec. 3.2,
+    "Sparse Evidence Probing", Eq. 1 and the block-sparse attention it cites);
+  * the frame-aligned block partition, text tokens partitioned independently
+    (Appendix "Detailed Sparse Prefilling", the paragraph after Eq. 6);
+  * logits q k^T / sqrt(d) (Eq. 8) and row-wise normalisation (Eq. 11);
+  * head averaging and the query-frame cue A_qf (Sec. 3.2, "Evidence
+    Decomposition").
+Parity pins for each function live in ``tests/test_oracle_pins.py``.
+"""
+from .attention import (  # noqa: F401
+    token_layout, allowed_row, probe_rows, probe, text_probabilities, evidence,
+)

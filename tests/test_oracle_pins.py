@@ -1,0 +1,340 @@
+"""Pins of the float64 oracle against facts other than itself (CPU only).
+
+Each test names the pin it realises:
+  golden  hand-derived example (tests/golden/hand_mask_example.json)
+  O1  closed form for constant keys
+  O2  row mass 1 and mass conservation of the evidence maps (also sharp logits)
+  O3  all-causal-tiles mask equals dense causal attention (torch SDPA, float64)
+  O4  brute force, pure-Python loops, tiny varlen inputs with random masks
+  O5  key-shift invariance of P, LSE shift by scale q.c
+  O6  GQA equals MHA with replicated KV heads
+  O7  packed varlen equals per-video runs
+  O8  reductions: frame, head, A_qf from tok
+  O9  planted frames rank top on the head-summed frame map
+  O10 linearity of O in V
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_05780_gb300 import workloads as wl
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _random_case(seed, videos=((6, 5), (10, 7)), hq=4, hkv=2, d=8, tile=4, npf=2, density=0.5,
+                 sharp=False):
+    """Tiny varlen case: videos = ((n_vis, n_text), ...); random valid CSR."""
+    rng = np.random.default_rng(seed)
+    n_vis = np.array([a for a, _ in videos], np.int32)
+    lens = np.array([a + b for a, b in videos])
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    n = int(cu[-1])
+    sc = 1.0 if sharp else 1.0 / math.sqrt(d)
+    q = wl.bf16_round(rng.standard_normal((n, hq, d)).astype(np.float32) * sc)
+    k = wl.bf16_round(rng.standard_normal((n, hkv, d)).astype(np.float32) * sc)
+    v = wl.bf16_round(rng.standard_normal((n, hkv, d)).astype(np.float32))
+    row_ptr, cols = [0], []
+    for nv in n_vis:
+        for r in range(-(-int(nv) // tile)):
+            kept = {r} | {c for c in range(r) if rng.random() < density}
+            cols += sorted(kept)
+            row_ptr.append(len(cols))
+    return dict(q=q, k=k, v=v, cu=cu, n_vis=n_vis, tile=tile, npf=npf,
+                row_ptr=np.array(row_ptr, np.int32), col_idx=np.array(cols, np.int32))
+
+
+def _run(c, scale=None):
+    o, lse = oracle.probe(c["q"], c["k"], c["v"], c["cu"], c["n_vis"], c["tile"], c["row_ptr"], c["col_idx"],
+                          scale=scale)
+    maps = oracle.evidence(c["q"], c["k"], c["cu"], c["n_vis"], c["npf"], scale=scale)
+    return o, lse, maps
+
+
+# ---------------------------------------------------------------- golden
+def test_golden_hand_example():
+    g = json.load(open(os.path.join(GOLDEN, "hand_mask_example.json")))
+    n = len(g["q"])
+    q = np.array(g["q"], np.float64).reshape(n, 1, 1)
+    k = np.log(np.array(g["k_exp"], np.float64)).reshape(n, 1, 1)
+    v = np.array(g["v"], np.float64).reshape(n, 1, 1)
+    cu = np.array([0, n]); n_vis = np.array([4])
+    o, lse = oracle.probe(q, k, v, cu, n_vis, g["tile"], np.array(g["row_ptr"]), np.array(g["col_idx"]),
+                          scale=1.0)
+    np.testing.assert_allclose(o[:, 0, 0], g["expected_o"], rtol=1e-14, atol=1e-14)
+    np.testing.assert_allclose(lse[0], np.log(g["expected_lse_exp"]), rtol=1e-14, atol=1e-14)
+    tok, frame, head, aqf = oracle.evidence(q, k, cu, n_vis, g["tokens_per_frame"], scale=1.0)
+    np.testing.assert_allclose(tok[0], g["expected_tok"], rtol=1e-13)
+    np.testing.assert_allclose(frame[0], g["expected_frame"], rtol=1e-13)
+    np.testing.assert_allclose(head[0], g["expected_head"], rtol=1e-13)
+    np.testing.assert_allclose(aqf, g["expected_aqf"], rtol=1e-13)
+
+
+def test_golden_layout_rule():
+    # text tiles restart at the text start: n_vis = 5, tile 4 -> visual tiles {0-3} {4}; text {5-8} {9}
+    is_text, tid = oracle.token_layout(5, 5, 4)
+    assert list(tid) == [0, 0, 0, 0, 1, 2, 2, 2, 2, 3]
+    assert list(is_text) == [False] * 5 + [True] * 5
+
+
+# ---------------------------------------------------------------- O1
+def _allowed_count_sink_window(p, n_vis, tile, window):
+    """|allowed(p)| for the sink + causal-window mask, counted from tile lengths."""
+    if p >= n_vis:
+        return p + 1
+    r = p // tile
+    tiles = ({0} | set(range(max(0, r - window + 1), r))) - {r}
+    return sum(min(tile, n_vis - t * tile) for t in tiles) + (p - r * tile + 1)
+
+
+@pytest.mark.parametrize("window", [1, 2, 3])
+def test_O1_constant_keys(window):
+    rng = np.random.default_rng(11)
+    n_vis, n_text, tile, d = 22, 9, 4, 8          # ragged last visual tile (22 = 5*4 + 2)
+    n = n_vis + n_text
+    cfg = wl.ProbeConfig("t", (11,), 2, (n_text,), 2, 1, d, tile, window)
+    row_ptr, col_idx = wl.build_mask(cfg)
+    q = rng.standard_normal((n, 2, d))
+    kvec = rng.standard_normal(d)
+    k = np.broadcast_to(kvec, (n, 1, d)).copy()
+    v = rng.standard_normal((n, 1, d))
+    cu = np.array([0, n]); nv = np.array([n_vis])
+    scale = 0.37
+    o, lse = oracle.probe(q, k, v, cu, nv, tile, row_ptr, col_idx, scale=scale)
+    for p in range(n):
+        cnt = _allowed_count_sink_window(p, n_vis, tile, window)
+        for h in range(2):
+            assert abs(lse[h, p] - (scale * q[p, h] @ kvec + math.log(cnt))) < 1e-12
+    # O_i is the mean of the allowed values: check against explicit tile arithmetic for a few rows
+    p = n_vis - 1                                   # last visual row, ragged tile 5
+    r = p // tile
+    idx = [j for t in sorted({0} | set(range(max(0, r - window + 1), r + 1)))
+           for j in range(t * tile, min((t + 1) * tile, n_vis)) if j <= p]
+    np.testing.assert_allclose(o[p, 0], v[idx, 0].mean(axis=0), atol=1e-13)
+    np.testing.assert_allclose(o[n - 1, 1], v[:, 0].mean(axis=0), atol=1e-13)
+    # evidence with constant keys: P = 1/(p+1) on each text row p
+    tok, frame, head, aqf = oracle.evidence(q, k, cu, nv, 2, scale=scale)
+    expect = sum(1.0 / (p + 1) for p in range(n_vis, n))
+    np.testing.assert_allclose(tok, expect, rtol=1e-13)
+    np.testing.assert_allclose(aqf, 2 * expect / n_text, rtol=1e-13)
+
+
+# ---------------------------------------------------------------- O2
+@pytest.mark.parametrize("sharp", [False, True])
+def test_O2_row_mass(sharp):
+    c = _random_case(2, sharp=sharp)
+    hq = c["q"].shape[1]
+    for b in range(2):
+        nv = int(c["n_vis"][b]); n_text = int(c["cu"][b + 1] - c["cu"][b]) - nv
+        for h in range(hq):
+            p = oracle.text_probabilities(c["q"], c["k"], c["cu"], c["n_vis"], b, h)
+            assert np.all(np.isfinite(p))
+            np.testing.assert_allclose(p.sum(axis=1), 1.0, atol=1e-12)
+    tok, frame, head, aqf = oracle.evidence(c["q"], c["k"], c["cu"], c["n_vis"], c["npf"])
+    for b in range(2):
+        nv = int(c["n_vis"][b]); n_text = int(c["cu"][b + 1] - c["cu"][b]) - nv
+        for h in range(hq):
+            p = oracle.text_probabilities(c["q"], c["k"], c["cu"], c["n_vis"], b, h)
+            text_mass = p[:, nv:].sum()
+            assert abs(head[b, h] + text_mass - n_text) < 1e-10
+    if sharp:
+        # large logits: rows must still normalise; LSE finite and above the row max
+        o, lse, _ = _run(c)
+        assert np.all(np.isfinite(o)) and np.all(np.isfinite(lse))
+
+
+# ---------------------------------------------------------------- O3
+def test_O3_all_tiles_equals_dense_causal_sdpa():
+    torch = pytest.importorskip("torch")
+    c = _random_case(3, videos=((12, 6), (10, 4)), density=1.0)
+    o, lse, _ = _run(c)
+    hq, hkv = c["q"].shape[1], c["k"].shape[1]
+    for b in range(2):
+        s0, s1 = int(c["cu"][b]), int(c["cu"][b + 1])
+        qt = torch.from_numpy(c["q"][s0:s1].astype(np.float64)).transpose(0, 1)       # [H, n, d]
+        kt = torch.from_numpy(c["k"][s0:s1].astype(np.float64)).transpose(0, 1).repeat_interleave(hq // hkv, 0)
+        vt = torch.from_numpy(c["v"][s0:s1].astype(np.float64)).transpose(0, 1).repeat_interleave(hq // hkv, 0)
+        ref = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True)
+        np.testing.assert_allclose(o[s0:s1], ref.transpose(0, 1).numpy(), atol=1e-12)
+
+
+# ---------------------------------------------------------------- O4
+def _brute(c, scale):
+    """Pure-Python loops straight from the position rules."""
+    q, k, v, cu, n_vis, tile = c["q"], c["k"], c["v"], c["cu"], c["n_vis"], c["tile"]
+    n, hq, d = q.shape
+    hkv = k.shape[1]
+    o = [[[0.0] * d for _ in range(hq)] for _ in range(n)]
+    lse = [[0.0] * n for _ in range(hq)]
+    row = 0
+    sets = []
+    for b in range(len(n_vis)):
+        vs = []
+        for _ in range(-(-int(n_vis[b]) // tile)):
+            vs.append(set(int(x) for x in c["col_idx"][c["row_ptr"][row]:c["row_ptr"][row + 1]]))
+            row += 1
+        sets.append(vs)
+    for b in range(len(n_vis)):
+        s0, s1, nv = int(cu[b]), int(cu[b + 1]), int(n_vis[b])
+        for i in range(s0, s1):
+            pi = i - s0
+            js = []
+            for j in range(s0, i + 1):
+                pj = j - s0
+                if pi >= nv or (pj // tile) in sets[b][pi // tile]:
+                    js.append(j)
+            for h in range(hq):
+                g = h * hkv // hq
+                logits = [scale * sum(float(q[i, h, e]) * float(k[j, g, e]) for e in range(d)) for j in js]
+                mx = max(logits)
+                z = sum(math.exp(x - mx) for x in logits)
+                lse[h][i] = mx + math.log(z)
+                for e in range(d):
+                    o[i][h][e] = sum(math.exp(x - lse[h][i]) * float(v[j, g, e]) for x, j in zip(logits, js))
+    return np.array(o), np.array(lse)
+
+
+@pytest.mark.parametrize("seed,tile,npf", [(4, 4, 2), (5, 8, 4), (6, 4, 4)])
+def test_O4_brute_force(seed, tile, npf):
+    c = _random_case(seed, videos=((8, 5), (16, 7), (4, 3)), tile=tile, npf=npf, d=6)
+    o, lse, (tok, frame, head, aqf) = _run(c)
+    scale = 1.0 / math.sqrt(6)
+    ob, lb = _brute(c, scale)
+    np.testing.assert_allclose(o, ob, atol=1e-12)
+    np.testing.assert_allclose(lse, lb, atol=1e-12)
+    # evidence by loops: text rows of each video onto its visual tokens
+    q, k = c["q"], c["k"]
+    hq, hkv = q.shape[1], k.shape[1]
+    vis_off = 0
+    for b in range(3):
+        s0, s1, nv = int(c["cu"][b]), int(c["cu"][b + 1]), int(c["n_vis"][b])
+        for h in range(hq):
+            g = h * hkv // hq
+            for m in range(nv):
+                acc = 0.0
+                for i in range(s0 + nv, s1):
+                    x = scale * sum(float(q[i, h, e]) * float(k[s0 + m, g, e]) for e in range(6))
+                    acc += math.exp(x - lb[h][i])
+                assert abs(tok[h, vis_off + m] - acc) < 1e-12
+        vis_off += nv
+
+
+# ---------------------------------------------------------------- O5
+def test_O5_key_shift_invariance():
+    c = _random_case(7)
+    o, lse, maps = _run(c)
+    shift = np.random.default_rng(1).standard_normal(c["k"].shape[2])
+    c2 = dict(c)
+    c2["k"] = c["k"].astype(np.float64) + shift               # same shift for every key and KV head
+    o2, lse2, maps2 = _run(c2)
+    np.testing.assert_allclose(o2, o, atol=1e-12)
+    scale = 1.0 / math.sqrt(c["q"].shape[2])
+    np.testing.assert_allclose(lse2, lse + scale * (c["q"].astype(np.float64) @ shift).T, atol=1e-12)
+    for a, b in zip(maps, maps2):
+        np.testing.assert_allclose(a, b, atol=1e-12)
+
+
+# ---------------------------------------------------------------- O6
+def test_O6_gqa_equals_replicated_mha():
+    c = _random_case(8, hq=6, hkv=2)
+    o, lse, maps = _run(c)
+    c2 = dict(c)
+    c2["k"] = np.repeat(c["k"], 3, axis=1)          # KV head g serves query heads 3g..3g+2
+    c2["v"] = np.repeat(c["v"], 3, axis=1)
+    o2, lse2, maps2 = _run(c2)
+    np.testing.assert_array_equal(o2, o)
+    np.testing.assert_array_equal(lse2, lse)
+    for a, b in zip(maps, maps2):
+        np.testing.assert_array_equal(a, b)
+
+
+# ---------------------------------------------------------------- O7
+def test_O7_varlen_independence():
+    c = _random_case(9, videos=((8, 3), (12, 6), (4, 2)))
+    o, lse, (tok, frame, head, aqf) = _run(c)
+    row = 0
+    vis0 = fr0 = 0
+    for b in range(3):
+        s0, s1, nv = int(c["cu"][b]), int(c["cu"][b + 1]), int(c["n_vis"][b])
+        nvt = -(-nv // c["tile"])
+        rp = c["row_ptr"][row:row + nvt + 1] - c["row_ptr"][row]
+        ci = c["col_idx"][c["row_ptr"][row]:c["row_ptr"][row + nvt]]
+        row += nvt
+        one = dict(q=c["q"][s0:s1], k=c["k"][s0:s1], v=c["v"][s0:s1], cu=np.array([0, s1 - s0]),
+                   n_vis=np.array([nv]), tile=c["tile"], npf=c["npf"], row_ptr=rp, col_idx=ci)
+        ob, lb, (tb, fb, hb, ab) = _run(one)
+        np.testing.assert_array_equal(ob, o[s0:s1])
+        np.testing.assert_array_equal(lb, lse[:, s0:s1])
+        nf = nv // c["npf"]
+        np.testing.assert_array_equal(tb, tok[:, vis0:vis0 + nv])
+        np.testing.assert_array_equal(fb, frame[:, fr0:fr0 + nf])
+        np.testing.assert_array_equal(hb[0], head[b])
+        np.testing.assert_array_equal(ab, aqf[fr0:fr0 + nf])
+        vis0 += nv; fr0 += nf
+
+
+# ---------------------------------------------------------------- O8
+def test_O8_reductions():
+    c = _random_case(10, videos=((8, 3), (12, 6)), npf=4)
+    tok, frame, head, aqf = oracle.evidence(c["q"], c["k"], c["cu"], c["n_vis"], 4)
+    hq = c["q"].shape[1]
+    vis0 = fr0 = 0
+    for b in range(2):
+        nv = int(c["n_vis"][b]); nf = nv // 4
+        n_text = int(c["cu"][b + 1] - c["cu"][b]) - nv
+        for t in range(nf):
+            for h in range(hq):
+                assert abs(frame[h, fr0 + t] - sum(tok[h, vis0 + 4 * t + u] for u in range(4))) < 1e-14
+            assert abs(aqf[fr0 + t] - sum(frame[h, fr0 + t] for h in range(hq)) / (hq * n_text)) < 1e-14
+        for h in range(hq):
+            assert abs(head[b, h] - frame[h, fr0:fr0 + nf].sum()) < 1e-13
+        assert aqf[fr0:fr0 + nf].sum() <= 1.0 + 1e-12
+        assert np.all(tok[:, vis0:vis0 + nv] >= 0)
+        vis0 += nv; fr0 += nf
+
+
+# ---------------------------------------------------------------- O9
+@pytest.mark.parametrize("name", ["tiny", "single"])
+def test_O9_planted_frames_rank_top(name):
+    p = wl.make_probe(wl.CONFIGS[name])
+    tok, frame, head, aqf = oracle.evidence(p.q, p.k, p.cu_seqlens, p.n_vis, p.cfg.tokens_per_frame)
+    planted = p.planted[0]
+    top = np.sort(np.argsort(-frame.sum(axis=0), kind="stable")[:planted.size])
+    np.testing.assert_array_equal(top, planted)
+    top_aqf = np.sort(np.argsort(-aqf, kind="stable")[:planted.size])
+    np.testing.assert_array_equal(top_aqf, planted)
+
+
+# ---------------------------------------------------------------- O10
+def test_O10_linearity_in_v():
+    c = _random_case(12)
+    rng = np.random.default_rng(5)
+    v2 = rng.standard_normal(c["v"].shape)
+    o1, _, _ = _run(c)
+    c2 = dict(c); c2["v"] = v2
+    o2, _, _ = _run(c2)
+    c3 = dict(c); c3["v"] = 2.5 * c["v"].astype(np.float64) - 0.75 * v2
+    o3, _, _ = _run(c3)
+    np.testing.assert_allclose(o3, 2.5 * o1 - 0.75 * o2, atol=1e-12)
+
+
+# ---------------------------------------------------------------- planted mistakes
+def test_pins_catch_planted_mistakes(monkeypatch):
+    """A wrong mask rule or a wrong GQA grouping in the oracle must fail a pin."""
+    import oracle.attention as op
+    g = json.load(open(os.path.join(GOLDEN, "hand_mask_example.json")))
+    n = len(g["q"])
+    q = np.ones((n, 1, 1)); k = np.log(np.array(g["k_exp"], float)).reshape(n, 1, 1)
+    v = np.array(g["v"], float).reshape(n, 1, 1)
+    good = op.allowed_row
+
+    def ignores_mask(p, is_text, tile_id, retained):       # planted mistake: dense causal rows
+        return good(p, np.ones_like(is_text), tile_id, retained)
+    monkeypatch.setattr(op, "allowed_row", ignores_mask)
+    o, _ = op.probe(q, k, v, np.array([0, n]), np.array([4]), 2, np.array(g["row_ptr"]),
+                    np.array(g["col_idx"]), scale=1.0)
+    assert not np.allclose(o[:, 0, 0], g["expected_o"])
