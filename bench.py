@@ -1,0 +1,405 @@
+"""Benchmark of the sparse-prefill evidence probe on one GB300 (or N replicas).
+
+One step = the whole hot path on one batch: evisel_probe_attention (block-sparse
+GQA attention + split-KV merge, text-logit spill) and evisel_evidence_reduce
+(token / frame / head maps and A_qf). Default workload: the 65,664-token probe
+(1024 frames x 64 pooled tokens + 128 text tokens, 28 query / 4 KV heads,
+d = 128, 128-token tiles, sink + 16-tile window + 32 random tiles per visual
+row tile). Inputs are synthetic (seeded), resident in HBM when the timed region
+starts, and larger than L2, so no flush is needed between steps.
+
+Prints one JSON line (rank 0). --impl reference times the float64 oracle on
+the host cores instead (bounded sample of the same workload).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_05780_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "probe-attention TFLOP/s (unmasked) & % GB300 BF16 peak; evidence-map GB/s"
+
+
+def _env_int(name, default):
+    try:
+        return int(os.environ.get(name, default))
+    except ValueError:
+        return default
+
+
+def workload_stats(probe):
+    """Algorithmic work of one probe layer (kept tiles only, full-tile convention)."""
+    cfg = probe.cfg
+    T, d, hq = cfg.tile, cfg.head_dim, cfg.hq
+    elems = 0
+    valid = 0
+    tiles = 0
+    r = 0
+    for b in range(len(probe.n_vis)):
+        nv = int(probe.n_vis[b])
+        nt = int(probe.n_text[b])
+        n_vt, n_tt = -(-nv // T), -(-nt // T)
+        tl = lambda c, n: min(T, n - c * T)
+        for t in range(n_vt):
+            rows = tl(t, nv)
+            for c in probe.col_idx[probe.row_ptr[r]:probe.row_ptr[r + 1]]:
+                cols = tl(int(c), nv)
+                elems += rows * cols
+                valid += rows * cols if c != t else rows * (rows + 1) // 2
+                tiles += 1
+            r += 1
+        for t in range(n_tt):
+            rows = tl(t, nt)
+            for c in range(n_vt):
+                elems += rows * tl(c, nv); valid += rows * tl(c, nv); tiles += 1
+            for u in range(t + 1):
+                cols = tl(u, nt)
+                elems += rows * cols
+                valid += rows * cols if u != t else rows * (rows + 1) // 2
+                tiles += 1
+    flop = 4.0 * d * hq * elems
+    flop_valid = 4.0 * d * hq * valid
+    n_tok = int(probe.cu_seqlens[-1])
+    spill = sum(hq * int(nt) * int(nv) * 4 for nv, nt in zip(probe.n_vis, probe.n_text))
+    lse_read = sum(hq * int(nt) * 4 for nt in probe.n_text)
+    total_vis = int(np.sum(probe.n_vis))
+    frames = total_vis // cfg.tokens_per_frame
+    maps = 4 * (hq * total_vis + hq * frames + len(probe.n_vis) * hq + frames)
+    return dict(flop=flop, flop_valid=flop_valid, tiles=tiles, n_tok=n_tok, spill_bytes=spill,
+                evidence_bytes=spill + lse_read + maps, map_bytes=maps)
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        j = json.load(open(p))
+        return dict(hbm=j["hbm_gbs"], bf16=j["bf16_tflops"], bf16_sus=j["bf16_tflops_sustained"],
+                    sm_max=j.get("sm_max_mhz"), source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, sm_max=2070.0, source="fallback")
+
+
+def _kernel_sha():
+    h = hashlib.sha256()
+    for f in ("probe_attn.cu", "sm103_ptx.cuh", "evisel_internal.h"):
+        h.update(open(os.path.join(ROOT, "paper_2608_05780_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def _traffic(workload):
+    """DRAM bytes per launch of the attention kernel from the committed ncu summary, if current."""
+    path = os.path.join(ROOT, "profiles", "probe_attn_long65k_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    kv = {}
+    for line in open(path):
+        if ":" in line and not line.startswith("#"):
+            k, v = line.split(":", 1)
+            kv[k.strip()] = v.strip()
+    if kv.get("source_sha") != _kernel_sha() or kv.get("workload") != workload:
+        return None
+    try:
+        return float(kv["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.file = None
+
+    def start(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=self.file, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [r.split(",") for r in self.file.read().strip().splitlines() if r.count(",") >= 8]
+        os.unlink(self.file.name)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].strip() == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def _oracle_sample(probe, max_rows):
+    """Rows of the longest visual row tiles plus the text rows: a bounded slice of the workload."""
+    cfg = probe.cfg
+    T = cfg.tile
+    counts = np.diff(probe.row_ptr)
+    order = np.argsort(-counts, kind="stable")
+    rows, flop = [], 0.0
+    s0, nv = int(probe.cu_seqlens[0]), int(probe.n_vis[0])
+    nt = int(probe.n_text[0])
+    text_rows = list(range(s0 + nv, s0 + nv + nt))
+    n_vt = -(-nv // T)
+    rows += text_rows
+    flop += 4.0 * cfg.head_dim * cfg.hq * nt * (nv + -(-nt // T) * T)
+    for r in order:
+        if len(rows) >= max_rows or r >= n_vt:
+            break
+        rl = min(T, nv - int(r) * T)
+        rows += list(range(s0 + int(r) * T, s0 + int(r) * T + rl))
+        flop += 4.0 * cfg.head_dim * cfg.hq * rl * int(counts[r]) * T
+    return np.array(rows), flop
+
+
+def run_oracle(probe, max_rows):
+    import oracle
+    rows, flop = _oracle_sample(probe, max_rows)
+    t0 = time.perf_counter()
+    oracle.probe_rows(probe.q, probe.k, probe.v, probe.cu_seqlens, probe.n_vis, probe.cfg.tile, probe.row_ptr,
+                      probe.col_idx, rows)
+    oracle.evidence(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, probe.cfg.tokens_per_frame)
+    dt = time.perf_counter() - t0
+    return flop, dt, len(rows)
+
+
+def bench_reference(args, cfg):
+    rank = _env_int("RANK", 0)
+    if rank != 0:
+        return 0
+    probe = wl.make_probe(cfg)
+    st = workload_stats(probe)
+    for _ in range(args.warmup):
+        run_oracle(probe, args.ref_rows)
+    flops, times, nrows = 0.0, 0.0, 0
+    for _ in range(args.steps):
+        f, dt, nrows = run_oracle(probe, args.ref_rows)
+        flops += f
+        times += dt
+    value = flops / times / 1e12
+    cores = os.cpu_count()
+    sample = (f"{nrows} query rows (the text rows plus the longest visual row tiles) of {cfg.name}, all "
+              f"{cfg.hq} heads, dense float64 rows, plus the full text-row evidence maps; FLOP counted "
+              f"over the rows' kept tiles")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * times / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": _config_dict(cfg, st),
+            "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def _config_dict(cfg, st):
+    return {"workload": f"{cfg.name}: {cfg.description}", "tokens": st["n_tok"], "kept_tiles": st["tiles"],
+            "layers": cfg.layers, "videos": cfg.num_videos, "hq": cfg.hq, "hkv": cfg.hkv,
+            "head_dim": cfg.head_dim, "tile": cfg.tile, "tokens_per_frame": cfg.tokens_per_frame,
+            "l2": "inputs larger than L2 (no flush)", "parallelism": "replicas"}
+
+
+def bench_ours(args, cfg):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2608_05780_gb300 as ev
+
+    world = _env_int("WORLD_SIZE", 1)
+    rank = _env_int("RANK", 0)
+    local = _env_int("LOCAL_RANK", 0)
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    ev.ensure_built()
+    probe = wl.make_probe(cfg)
+    st = workload_stats(probe)
+    q = torch.from_numpy(probe.q).cuda().to(torch.bfloat16)
+    k = torch.from_numpy(probe.k).cuda().to(torch.bfloat16)
+    v = torch.from_numpy(probe.v).cuda().to(torch.bfloat16)
+    n, hq, d = q.shape
+    o = torch.empty_like(q)
+    lse = torch.empty((hq, n), dtype=torch.float32, device="cuda")
+    total_vis = int(np.sum(probe.n_vis))
+    frames = total_vis // cfg.tokens_per_frame
+    maps = [torch.zeros((hq, total_vis), device="cuda"), torch.zeros((hq, frames), device="cuda"),
+            torch.zeros((len(probe.n_vis), hq), device="cuda"), torch.zeros((frames,), device="cuda")]
+    ws = ev.Workspace()
+    stream = torch.cuda.current_stream()
+
+    def step(ev_marks=None):
+        if ev_marks:
+            ev_marks[0].record(stream)
+        ev.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                  probe.row_ptr, probe.col_idx, ws=ws, o=o, lse=lse)
+        if ev_marks:
+            ev_marks[1].record(stream)
+        ev.evisel_evidence_reduce(ws, hq, probe.n_vis, cfg.tokens_per_frame, len(probe.n_vis), tok=maps[0],
+                                  frame=maps[1], head=maps[2], aqf=maps[3])
+        if ev_marks:
+            ev_marks[2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if ev.evisel_status(ws) != 0:
+        raise RuntimeError("device status reported an error")
+
+    marks = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        step(marks[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = t_start.elapsed_time(t_end)
+    attn_ms = [m[0].elapsed_time(m[1]) for m in marks]
+    ev_ms = [m[1].elapsed_time(m[2]) for m in marks]
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    ms_step = elapsed_ms / args.steps
+    value = world * st["flop"] / (ms_step * 1e-3) / 1e12
+    attn_avg = sum(attn_ms) / len(attn_ms)
+    ev_avg = sum(ev_ms) / len(ev_ms)
+    peaks = _peaks()
+    attn_tflops = st["flop"] / (attn_avg * 1e-3) / 1e12
+    ev_gbs = st["evidence_bytes"] / (ev_avg * 1e-3) / 1e9
+
+    # End to end through the public API with host buffers: pinned inputs copied in,
+    # evidence maps copied out, every step.
+    hq_, hk_, hv_ = (t.cpu().pin_memory() for t in (q, k, v))
+    host_maps = [m.cpu().pin_memory() for m in maps]
+    h2d = sum(t.numel() * t.element_size() for t in (hq_, hk_, hv_))
+    d2h = sum(m.numel() * m.element_size() for m in maps)
+
+    def e2e_step():
+        q.copy_(hq_, non_blocking=True)
+        k.copy_(hk_, non_blocking=True)
+        v.copy_(hv_, non_blocking=True)
+        step()
+        for hm, m in zip(host_maps, maps):
+            hm.copy_(m, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / args.steps
+    status = ev.evisel_status(ws)
+    ws.free()
+    if status != 0:
+        raise RuntimeError("device status reported an error")
+
+    line = None
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": _config_dict(cfg, st),
+                "frac_of_bf16_peak": value / world / peaks["bf16"],
+                "tokens_per_s": world * st["n_tok"] * cfg.layers / (ms_step * 1e-3),
+                "flop_per_step": st["flop"], "flop_causal_valid_per_step": st["flop_valid"],
+                "attention": {"ms": attn_avg, "tflops": attn_tflops, "frac_of_bf16_peak": attn_tflops / peaks["bf16"],
+                              "tflops_causal_valid": st["flop_valid"] / (attn_avg * 1e-3) / 1e12},
+                "evidence": {"ms": ev_avg, "gbs": ev_gbs, "frac_of_hbm": ev_gbs / peaks["hbm"],
+                             "bytes": st["evidence_bytes"]},
+                "roofline": {"bound": "tensor", "achieved": attn_tflops, "peak": peaks["bf16"], "unit": "TFLOP/s",
+                             "frac": attn_tflops / peaks["bf16"],
+                             "traffic": _traffic(cfg.name),
+                             "kernel": "probe_attn (evisel_probe_attention: probe_attn_kernel + attn_combine)",
+                             "peak_source": f"{peaks['source']} bf16 burst"},
+                "e2e": {"value": world * st["flop"] / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+                "gpu_launches": args.steps * (4 if _has_combine(probe) else 3),
+                "clocks": clk}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        flop, dt, nrows = run_oracle(probe, args.ref_rows)
+        line["cpu_baseline"] = {"value": flop / dt / 1e12, "unit": "TFLOP/s", "cores": os.cpu_count(),
+                                "kind": "oracle",
+                                "sample": f"{nrows} query rows (text rows + longest visual row tiles) of "
+                                          f"{cfg.name}, all heads, plus the full text-row evidence maps; "
+                                          f"{dt:.1f} s"}
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def _has_combine(probe):
+    cfg = probe.cfg
+    counts = np.diff(probe.row_ptr)
+    split = max(int(counts.max()) if counts.size else 1, 8)
+    for nv, nt in zip(probe.n_vis, probe.n_text):
+        n_vt, n_tt = -(-int(nv) // cfg.tile), -(-int(nt) // cfg.tile)
+        if n_tt and n_vt + n_tt > split:
+            return True
+    return False
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default="long65k", choices=sorted(wl.CONFIGS))
+    ap.add_argument("--ref-rows", type=int, default=256)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    cfg = wl.CONFIGS[args.config]
+    if args.impl == "reference":
+        return bench_reference(args, cfg)
+    return bench_ours(args, cfg)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,143 @@
+/*
+ * evisel.h - C ABI of the GB300 (sm_103a) sparse-prefill evidence probe.
+ *
+ * The probe is the paper's evidence-grounding pass (Sec. 3.2, "Sparse Evidence
+ * Probing", Eq. 1): block-sparse, causal, grouped-query prefill attention over
+ * a packed batch of videos, each laid out as X = [X_vis; X_Q] (pooled visual
+ * tokens, then the query's text tokens; Appendix "Detailed Sparse
+ * Prefilling"), followed by the attention evidence read off the text rows
+ * (Sec. 3.2, "Evidence Decomposition"): the softmax mass from the text rows
+ * onto every visual token, reduced per token, per frame and per head, and the
+ * query-frame cue A_qf.
+ *
+ * Conventions for every entry point:
+ *   - Pointers marked "device" are CUDA device pointers owned by the caller;
+ *     pointers marked "host" are ordinary host memory read during the call only.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     All device work is enqueued asynchronously on it; nothing blocks the host
+ *     except evisel_status() and evisel_free().
+ *   - Return value 0 = success, negative = an EVISEL_E* code below; on failure
+ *     nothing has been enqueued and evisel_last_error() describes the cause
+ *     (thread-local string).
+ *   - Thread safety: calls are reentrant provided each thread uses its own
+ *     workspace.
+ */
+#ifndef EVISEL_H
+#define EVISEL_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define EVISEL_OK             0
+#define EVISEL_EINVAL        -1  /* null pointer, bad count, misaligned pointer   */
+#define EVISEL_EUNSUPPORTED  -2  /* head_dim, tile, hq % hkv or N_v outside the set */
+#define EVISEL_EMASK         -3  /* unsorted / out-of-range / non-causal CSR, missing diagonal */
+#define EVISEL_ECUDA         -4  /* a CUDA runtime/driver call failed             */
+#define EVISEL_ENOMEM        -5  /* device or pinned allocation failed            */
+#define EVISEL_ETIMEOUT      -6  /* device-side: a bounded wait gave up           */
+#define EVISEL_EBOUNDS       -7  /* device-side: an index check failed            */
+#define EVISEL_ESTATE        -8  /* evidence requested before any probe on the workspace */
+
+/* Opaque workspace owned by the library: work list, device copy of the mask,
+ * split-KV partials and the text-row logit spill. Created by the first
+ * evisel_probe_attention() call that receives *ws == NULL; reused (grown if
+ * needed) by later calls; released only by evisel_free(). */
+typedef struct evisel_ws evisel_ws;
+
+/* Description of one probe call (one transformer layer).
+ *
+ * Token layout (Appendix, "Detailed Sparse Prefilling"): videos are packed back
+ * to back; video b spans global tokens [cu_seqlens[b], cu_seqlens[b+1]), its
+ * first n_vis[b] tokens are visual (n_vis[b] = T_b * tokens_per_frame), the rest
+ * are its text tokens. Visual tokens are cut into tiles of `tile` tokens from the
+ * visual start and text tokens independently from the text start; the last tile
+ * of each may be short. tile must be a multiple of tokens_per_frame so that no
+ * frame crosses a tile (Eq. 1: block boundaries align with frame boundaries).
+ *
+ * Mask (Sec. 3.2: block-sparse attention keeps only retained blocks): a CSR over
+ * the visual row tiles of all videos in video order; row r lists, sorted
+ * ascending, the video-local visual kv-tile ids its queries may attend to. Each
+ * row must contain its own (diagonal) tile and only tiles <= it. Text rows are
+ * implicitly dense and causal over their own video. Within a kept tile, keys are
+ * causal (key position <= query position).
+ *
+ * Softmax (Eq. 8, Eq. 11): logits s_ij = softmax_scale * q_i . k_j with query
+ * head h reading KV head h / (hq / hkv); LSE_i = ln sum_j exp(s_ij).
+ */
+typedef struct {
+  int32_t num_videos;            /* B >= 1                                         */
+  const int32_t* cu_seqlens_h;   /* host [B+1], cu_seqlens[0] = 0, non-decreasing   */
+  const int32_t* n_vis_h;        /* host [B], 0 <= n_vis[b] <= seqlen_b, a multiple of
+                                    tokens_per_frame; a video may have no text tokens
+                                    (its evidence is then zero) or no visual tokens  */
+  int32_t tokens_per_frame;      /* N_v: a power of two, 4 <= N_v <= tile          */
+  int32_t hq;                    /* query heads                                     */
+  int32_t hkv;                   /* KV heads, hq % hkv == 0                         */
+  int32_t head_dim;              /* d in {64, 128}                                  */
+  int32_t tile;                  /* t_s in {64, 128}                                */
+  float softmax_scale;           /* 0 => 1/sqrt(head_dim)                           */
+  const void* q;                 /* device bf16 [N_tot, hq, d], contiguous, 16-B aligned */
+  const void* k;                 /* device bf16 [N_tot, hkv, d]                     */
+  const void* v;                 /* device bf16 [N_tot, hkv, d]                     */
+  const int32_t* mask_row_ptr_h; /* host [R+1], R = sum_b ceil(n_vis[b] / tile)      */
+  const int32_t* mask_col_idx_h; /* host [row_ptr[R]]                               */
+  void* o;                       /* device bf16 [N_tot, hq, d] (written)            */
+  float* lse;                    /* device fp32 [hq, N_tot], natural log (written); must
+                                    stay alive until evisel_evidence_reduce() ran  */
+} evisel_probe_args;
+
+/* Block-sparse causal GQA varlen attention (Eq. 1; Appendix Eq. 8 and Eq. 11
+ * with exact token logits on every kept tile). Writes O and LSE for every
+ * token, and spills the text rows' logits onto their video's visual tokens into
+ * the workspace for evisel_evidence_reduce().
+ *   args      : the call description above (host struct, read during the call).
+ *   stream    : cudaStream_t as void*.
+ *   ws_inout  : in/out. *ws_inout == NULL -> a workspace is created and stored;
+ *               otherwise it is reused (grown when too small). The caller must not
+ *               use one workspace from two streams concurrently.
+ * Errors: EVISEL_EINVAL, EVISEL_EUNSUPPORTED, EVISEL_EMASK (validated on the host
+ * before any launch), EVISEL_ENOMEM, EVISEL_ECUDA. Device-side timeouts surface
+ * through evisel_status(). */
+int evisel_probe_attention(const evisel_probe_args* args, void* stream, evisel_ws** ws_inout);
+
+/* Evidence reduction over the text rows of the last probe on `ws` (Sec. 3.2,
+ * "Evidence Decomposition"; head averaging and the query-frame cue A_qf):
+ *   tok[h, m]   = sum_{text rows i} exp(s_im - LSE_i)      device fp32 [hq, sum_b n_vis[b]]
+ *   frame[h, t] = sum_{m in frame t} tok[h, m]             device fp32 [hq, sum_b T_b]
+ *   head[b, h]  = sum_{t in video b} frame[h, t]           device fp32 [B, hq]
+ *   aqf[t]      = sum_h frame[h, t] / (hq * n_text_b)      device fp32 [sum_b T_b]
+ *                 (0 for a video without text tokens)
+ * Columns of tok and frame are the videos' visual tokens / frames in video order.
+ * accumulate != 0 adds tok and frame into the existing contents (sum over
+ * layers); head and aqf are always recomputed from the resulting frame map, so
+ * they accumulate too. Must be enqueued on the probe's stream (or after it).
+ * Errors: EVISEL_EINVAL, EVISEL_ESTATE, EVISEL_ECUDA. */
+int evisel_evidence_reduce(const evisel_ws* ws, float* tok, float* frame, float* head, float* aqf,
+                           int accumulate, void* stream);
+
+/* Synchronises the stream of the workspace's last call, releases every device
+ * and host buffer of the workspace. NULL-safe. */
+void evisel_free(evisel_ws* ws);
+
+/* Synchronises the stream of the workspace's last call and returns the device
+ * status word (EVISEL_OK, EVISEL_ETIMEOUT or EVISEL_EBOUNDS), then clears it.
+ * Returns EVISEL_ECUDA if the synchronisation itself failed. */
+int evisel_status(evisel_ws* ws);
+
+/* Static description of a status code. */
+const char* evisel_strerror(int code);
+
+/* Detail of the last failure on the calling thread ("" if none). */
+const char* evisel_last_error(void);
+
+/* Bytes of device memory currently held by the workspace (0 for NULL). */
+int64_t evisel_workspace_bytes(const evisel_ws* ws);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EVISEL_H */

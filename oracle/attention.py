@@ -26,7 +26,8 @@ Evidence (Sec. 3.2, "Evidence Decomposition"): with P from the text rows,
   frame[h, t] = sum of tok[h, m] over frame t's N_v tokens [t N_v, (t+1) N_v)
   head[b, h]  = sum over the video's frames of frame[h, t]
   A_qf[t]     = sum_h frame[h, t] / (Hq * n_text)   (average over the whole
-                query-token group and over heads)
+                query-token group and over heads; 0 for a video without query
+                tokens, a case the paper does not have)
 """
 from __future__ import annotations
 
@@ -175,5 +176,6 @@ def evidence(q, k, cu_seqlens, n_vis, tokens_per_frame, scale=None):
             f_map = t_map.reshape(int(frames[b]), tokens_per_frame).sum(axis=1)
             frame[h, fr_off[b]:fr_off[b + 1]] = f_map
             head[b, h] = f_map.sum()
-        aqf[fr_off[b]:fr_off[b + 1]] = frame[:, fr_off[b]:fr_off[b + 1]].sum(axis=0) / (hq * n_text)
+        if n_text > 0:      # a video without query tokens carries no query-frame evidence
+            aqf[fr_off[b]:fr_off[b + 1]] = frame[:, fr_off[b]:fr_off[b + 1]].sum(axis=0) / (hq * n_text)
     return tok, frame, head, aqf

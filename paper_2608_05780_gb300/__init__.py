@@ -1,0 +1,16 @@
+"""GB300-native (sm_103a) sparse-prefill evidence probe.
+
+The product is ``libevisel.so`` (C ABI in ``include/evisel.h``); this package
+holds its sources (``csrc/``), the in-tree build and a thin ctypes binding with
+the same entry-point names. ``workloads`` draws the seeded synthetic inputs.
+"""
+from ._binding import (  # noqa: F401
+    EviselError, Workspace, evisel_evidence_reduce, evisel_free, evisel_probe_attention, evisel_status, load,
+)
+
+
+def ensure_built():
+    """Builds the library if needed and loads it."""
+    from .build import build
+    build()
+    return load()

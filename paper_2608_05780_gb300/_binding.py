@@ -1,0 +1,199 @@
+"""ctypes binding of libevisel.so: argument marshalling only.
+
+The functions carry the C ABI's names (include/evisel.h). PyTorch provides
+device memory and the current CUDA stream; every step of the probe runs in the
+library's sm_103a kernels. There is no CPU fallback: if the library cannot be
+loaded the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libevisel.so")
+
+EVISEL_OK = 0
+_ERRORS = {-1: "EINVAL", -2: "EUNSUPPORTED", -3: "EMASK", -4: "ECUDA", -5: "ENOMEM", -6: "ETIMEOUT",
+           -7: "EBOUNDS", -8: "ESTATE"}
+
+
+class EviselError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"{_ERRORS.get(code, code)} ({code}): {msg}")
+        self.code = code
+
+
+class ProbeArgs(ctypes.Structure):
+    _fields_ = [
+        ("num_videos", ctypes.c_int32),
+        ("cu_seqlens_h", ctypes.POINTER(ctypes.c_int32)),
+        ("n_vis_h", ctypes.POINTER(ctypes.c_int32)),
+        ("tokens_per_frame", ctypes.c_int32),
+        ("hq", ctypes.c_int32),
+        ("hkv", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32),
+        ("tile", ctypes.c_int32),
+        ("softmax_scale", ctypes.c_float),
+        ("q", ctypes.c_void_p),
+        ("k", ctypes.c_void_p),
+        ("v", ctypes.c_void_p),
+        ("mask_row_ptr_h", ctypes.POINTER(ctypes.c_int32)),
+        ("mask_col_idx_h", ctypes.POINTER(ctypes.c_int32)),
+        ("o", ctypes.c_void_p),
+        ("lse", ctypes.c_void_p),
+    ]
+
+
+EXPORTS = ["evisel_probe_attention", "evisel_evidence_reduce", "evisel_free", "evisel_status",
+           "evisel_strerror", "evisel_last_error", "evisel_workspace_bytes"]
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Loads the library (once) and declares the C signatures."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"libevisel.so is not built ({path}); run paper_2608_05780_gb300.build.build()")
+    lib = ctypes.CDLL(path)
+    vp, i32 = ctypes.c_void_p, ctypes.c_int
+    lib.evisel_probe_attention.argtypes = [ctypes.POINTER(ProbeArgs), vp, ctypes.POINTER(vp)]
+    lib.evisel_probe_attention.restype = i32
+    lib.evisel_evidence_reduce.argtypes = [vp, vp, vp, vp, vp, i32, vp]
+    lib.evisel_evidence_reduce.restype = i32
+    lib.evisel_free.argtypes = [vp]
+    lib.evisel_free.restype = None
+    lib.evisel_status.argtypes = [vp]
+    lib.evisel_status.restype = i32
+    lib.evisel_strerror.argtypes = [i32]
+    lib.evisel_strerror.restype = ctypes.c_char_p
+    lib.evisel_last_error.argtypes = []
+    lib.evisel_last_error.restype = ctypes.c_char_p
+    lib.evisel_workspace_bytes.argtypes = [vp]
+    lib.evisel_workspace_bytes.restype = ctypes.c_int64
+    _lib = lib
+    return lib
+
+
+def _check(rc):
+    if rc != EVISEL_OK:
+        raise EviselError(rc, _lib.evisel_last_error().decode())
+
+
+def _i32(a):
+    arr = np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+    return arr, arr.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
+
+
+def _stream_handle(stream):
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+class Workspace:
+    """Owner of an evisel_ws* (freed with evisel_free)."""
+
+    def __init__(self):
+        self.ptr = ctypes.c_void_p(None)
+
+    @property
+    def nbytes(self):
+        return int(load().evisel_workspace_bytes(self.ptr))
+
+    def free(self):
+        if self.ptr.value:
+            load().evisel_free(self.ptr)
+            self.ptr = ctypes.c_void_p(None)
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
+              softmax_scale=0.0):
+    """Fills the C struct; returns (struct, keepalive) - keepalive holds the host arrays."""
+    cu, cu_p = _i32(cu_seqlens)
+    nv, nv_p = _i32(n_vis)
+    rp, rp_p = _i32(row_ptr)
+    ci, ci_p = _i32(col_idx if len(col_idx) else np.zeros(1, np.int32))
+    a = ProbeArgs()
+    a.num_videos = len(nv)
+    a.cu_seqlens_h = cu_p
+    a.n_vis_h = nv_p
+    a.tokens_per_frame = int(tokens_per_frame)
+    a.hq = int(q.shape[1])
+    a.hkv = int(k.shape[1])
+    a.head_dim = int(q.shape[2])
+    a.tile = int(tile)
+    a.softmax_scale = float(softmax_scale)
+    a.q, a.k, a.v = q.data_ptr(), k.data_ptr(), v.data_ptr()
+    a.mask_row_ptr_h = rp_p
+    a.mask_col_idx_h = ci_p
+    a.o, a.lse = o.data_ptr(), lse.data_ptr()
+    return a, (cu, nv, rp, ci)
+
+
+def evisel_probe_attention(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx,
+                           ws=None, o=None, lse=None, softmax_scale=0.0, stream=None):
+    """Block-sparse GQA varlen probe attention. q/k/v: CUDA bf16 [N, H, d].
+
+    Returns (o [N, hq, d] bf16, lse [hq, N] fp32, ws).
+    """
+    import torch
+    lib = load()
+    for t in (q, k, v):
+        if not (t.is_cuda and t.dtype == torch.bfloat16 and t.is_contiguous() and t.dim() == 3):
+            raise ValueError("q, k, v must be contiguous CUDA bf16 tensors [N, H, d]")
+    n, hq, d = q.shape
+    if o is None:
+        o = torch.empty((n, hq, d), dtype=torch.bfloat16, device=q.device)
+    if lse is None:
+        lse = torch.empty((hq, n), dtype=torch.float32, device=q.device)
+    if ws is None:
+        ws = Workspace()
+    args, keep = make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
+                           softmax_scale)
+    _check(lib.evisel_probe_attention(ctypes.byref(args), _stream_handle(stream), ctypes.byref(ws.ptr)))
+    del keep
+    return o, lse, ws
+
+
+def evisel_evidence_reduce(ws, hq, n_vis, tokens_per_frame, num_videos, tok=None, frame=None, head=None,
+                           aqf=None, accumulate=False, stream=None, device="cuda"):
+    """Token / frame / head / A_qf evidence of the last probe on ``ws``.
+
+    Returns (tok [hq, sum n_vis], frame [hq, sum T], head [B, hq], aqf [sum T]).
+    """
+    import torch
+    lib = load()
+    total_vis = int(np.sum(n_vis))
+    total_frames = total_vis // int(tokens_per_frame)
+    f32 = dict(dtype=torch.float32, device=device)
+    if tok is None:
+        tok = torch.zeros((hq, total_vis), **f32)
+    if frame is None:
+        frame = torch.zeros((hq, total_frames), **f32)
+    if head is None:
+        head = torch.zeros((num_videos, hq), **f32)
+    if aqf is None:
+        aqf = torch.zeros((total_frames,), **f32)
+    _check(lib.evisel_evidence_reduce(ws.ptr, tok.data_ptr(), frame.data_ptr(), head.data_ptr(),
+                                      aqf.data_ptr(), int(bool(accumulate)), _stream_handle(stream)))
+    return tok, frame, head, aqf
+
+
+def evisel_status(ws):
+    return int(load().evisel_status(ws.ptr))
+
+
+def evisel_free(ws):
+    ws.free()

@@ -1,0 +1,588 @@
+// Host side of the C ABI: argument and mask validation, work planning (one
+// item per query row tile x head block x kv range, longest first), the
+// workspace arena, TMA descriptor encoding and kernel launches.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include "../../include/evisel.h"
+#include "evisel_internal.h"
+
+using namespace evisel;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const std::string& msg) {
+  g_last_error = msg;
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+  return fail(EVISEL_ECUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 3-D bf16 tensor [tokens, heads, d] viewed as {d, heads, tokens}; box {64, 1, rows}.
+int encode_map(CUtensorMap* map, const void* base, int n_tok, int heads, int d, int rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return fail(EVISEL_ECUDA, "cuTensorMapEncodeTiled unavailable from the driver");
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(heads),
+                        static_cast<cuuint64_t>(std::max(n_tok, 1))};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(heads) * d * 2};
+  cuuint32_t box[3] = {64, 1, static_cast<cuuint32_t>(rows)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(EVISEL_ECUDA, "cuTensorMapEncodeTiled failed: " + std::to_string(r));
+  return EVISEL_OK;
+}
+
+// Host-side plan of one probe call.
+struct Plan {
+  std::vector<WorkItem> items;
+  std::vector<KvTile> kv;
+  std::vector<VideoInfo> videos;
+  std::vector<CombineGroup> groups;
+  std::vector<EvChunk> chunks;
+  int n_parts = 0;
+  int64_t spill_floats = 0;
+  int total_vis = 0;
+  int total_frames = 0;
+  int n_tok = 0;
+};
+
+int validate(const evisel_probe_args* a) {
+  if (!a) return fail(EVISEL_EINVAL, "args is NULL");
+  if (a->num_videos < 0) return fail(EVISEL_EINVAL, "num_videos < 0");
+  if (a->num_videos > 0 && (!a->cu_seqlens_h || !a->n_vis_h))
+    return fail(EVISEL_EINVAL, "cu_seqlens_h / n_vis_h is NULL");
+  if (a->head_dim != 64 && a->head_dim != 128)
+    return fail(EVISEL_EUNSUPPORTED, "head_dim must be 64 or 128, got " + std::to_string(a->head_dim));
+  if (a->tile != 64 && a->tile != 128)
+    return fail(EVISEL_EUNSUPPORTED, "tile must be 64 or 128, got " + std::to_string(a->tile));
+  if (a->hq < 1 || a->hkv < 1) return fail(EVISEL_EINVAL, "hq and hkv must be >= 1");
+  if (a->hq % a->hkv != 0) return fail(EVISEL_EUNSUPPORTED, "hq must be a multiple of hkv");
+  const int npf = a->tokens_per_frame;
+  if (npf < 4 || npf > a->tile || (npf & (npf - 1)) != 0)
+    return fail(EVISEL_EUNSUPPORTED, "tokens_per_frame must be a power of two in [4, tile]");
+  if (!(a->softmax_scale >= 0.f) || !std::isfinite(a->softmax_scale))
+    return fail(EVISEL_EINVAL, "softmax_scale must be finite and >= 0");
+  if (a->num_videos == 0) return EVISEL_OK;
+  if (a->cu_seqlens_h[0] != 0) return fail(EVISEL_EINVAL, "cu_seqlens[0] must be 0");
+  int64_t rows = 0;
+  for (int b = 0; b < a->num_videos; ++b) {
+    const int64_t len = static_cast<int64_t>(a->cu_seqlens_h[b + 1]) - a->cu_seqlens_h[b];
+    if (len < 0) return fail(EVISEL_EINVAL, "cu_seqlens must be non-decreasing");
+    const int nv = a->n_vis_h[b];
+    if (nv < 0 || nv > len) return fail(EVISEL_EINVAL, "n_vis[" + std::to_string(b) + "] out of range");
+    if (nv % npf != 0) return fail(EVISEL_EINVAL, "n_vis must be a multiple of tokens_per_frame");
+    rows += (nv + a->tile - 1) / a->tile;
+  }
+  const int64_t n_tok = a->cu_seqlens_h[a->num_videos];
+  if (n_tok > (int64_t(1) << 30)) return fail(EVISEL_EINVAL, "too many tokens");
+  if (n_tok > 0) {
+    if (!a->q || !a->k || !a->v || !a->o || !a->lse) return fail(EVISEL_EINVAL, "a device pointer is NULL");
+    auto mis = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; };
+    if (mis(a->q) || mis(a->k) || mis(a->v) || mis(a->o) || mis(a->lse))
+      return fail(EVISEL_EINVAL, "device pointers must be 16-byte aligned");
+  }
+  if (rows > 0 && (!a->mask_row_ptr_h || !a->mask_col_idx_h)) return fail(EVISEL_EINVAL, "mask is NULL");
+  if (rows > 0) {
+    const int32_t* rp = a->mask_row_ptr_h;
+    const int32_t* ci = a->mask_col_idx_h;
+    if (rp[0] != 0) return fail(EVISEL_EMASK, "mask row_ptr[0] must be 0");
+    int64_t r = 0;
+    for (int b = 0; b < a->num_videos; ++b) {
+      const int n_vt = (a->n_vis_h[b] + a->tile - 1) / a->tile;
+      for (int t = 0; t < n_vt; ++t, ++r) {
+        const int32_t s = rp[r], e = rp[r + 1];
+        if (e <= s) return fail(EVISEL_EMASK, "mask row " + std::to_string(r) + " is empty");
+        for (int32_t i = s; i < e; ++i) {
+          const int32_t c = ci[i];
+          if (c < 0 || c > t)
+            return fail(EVISEL_EMASK, "mask row " + std::to_string(r) + " has non-causal or negative tile " +
+                                          std::to_string(c));
+          if (i > s && c <= ci[i - 1])
+            return fail(EVISEL_EMASK, "mask row " + std::to_string(r) + " is not strictly ascending");
+        }
+        if (ci[e - 1] != t)
+          return fail(EVISEL_EMASK, "mask row " + std::to_string(r) + " lacks its diagonal tile");
+      }
+    }
+  }
+  return EVISEL_OK;
+}
+
+void build_plan(const evisel_probe_args* a, Plan& P) {
+  const int T = a->tile;
+  const int hq = a->hq, gq = a->hq / a->hkv;
+  const int hp = 128 / T;                      // heads per CTA
+  P.n_tok = a->num_videos ? a->cu_seqlens_h[a->num_videos] : 0;
+
+  // Head blocks: consecutive heads of one KV group.
+  std::vector<int> head_blocks;
+  for (int g = 0; g < a->hkv; ++g)
+    for (int hh = 0; hh < gq; hh += hp) head_blocks.push_back(g * gq + hh);
+
+  // Videos.
+  int64_t spill = 0;
+  int vis_off = 0, frame_off = 0;
+  for (int b = 0; b < a->num_videos; ++b) {
+    VideoInfo v{};
+    v.vis_start = a->cu_seqlens_h[b];
+    v.n_vis = a->n_vis_h[b];
+    v.n_text = a->cu_seqlens_h[b + 1] - a->cu_seqlens_h[b] - v.n_vis;
+    v.vis_pitch = (v.n_vis + 3) & ~3;
+    v.spill_off = spill;
+    v.vis_off = vis_off;
+    v.frame_off = frame_off;
+    spill += static_cast<int64_t>(hq) * v.n_text * v.vis_pitch;
+    vis_off += v.n_vis;
+    frame_off += v.n_vis / a->tokens_per_frame;
+    P.videos.push_back(v);
+  }
+  P.spill_floats = spill;
+  P.total_vis = vis_off;
+  P.total_frames = frame_off;
+
+  // Visual row tiles: kv lists straight from the mask.
+  int max_visual = 1;
+  int64_t r = 0;
+  std::vector<WorkItem> items;
+  for (int b = 0; b < a->num_videos; ++b) {
+    const VideoInfo& v = P.videos[b];
+    const int n_vt = (v.n_vis + T - 1) / T;
+    for (int t = 0; t < n_vt; ++t, ++r) {
+      const int kv_begin = static_cast<int>(P.kv.size());
+      for (int32_t i = a->mask_row_ptr_h[r]; i < a->mask_row_ptr_h[r + 1]; ++i) {
+        const int c = a->mask_col_idx_h[i];
+        KvTile k{};
+        k.start = v.vis_start + c * T;
+        k.len = static_cast<int16_t>(std::min(T, v.n_vis - c * T));
+        k.diag = c == t;
+        k.visual = 1;
+        P.kv.push_back(k);
+      }
+      const int cnt = static_cast<int>(P.kv.size()) - kv_begin;
+      max_visual = std::max(max_visual, cnt);
+      for (int h : head_blocks) {
+        WorkItem it{};
+        it.q_start = v.vis_start + t * T;
+        it.q_len = std::min(T, v.n_vis - t * T);
+        it.head = h;
+        it.kv_begin = kv_begin;
+        it.kv_count = cnt;
+        it.part = -1;
+        it.video = b;
+        it.text_row0 = -1;
+        items.push_back(it);
+      }
+    }
+  }
+
+  // Text row tiles: dense causal over the video, split into chunks no longer
+  // than the longest visual row so that no CTA straggles.
+  const int split_len = std::max(max_visual, 8);
+  for (int b = 0; b < a->num_videos; ++b) {
+    const VideoInfo& v = P.videos[b];
+    const int n_vt = (v.n_vis + T - 1) / T;
+    const int n_tt = (v.n_text + T - 1) / T;
+    for (int t = 0; t < n_tt; ++t) {
+      const int kv_begin = static_cast<int>(P.kv.size());
+      for (int c = 0; c < n_vt; ++c) {
+        KvTile k{};
+        k.start = v.vis_start + c * T;
+        k.len = static_cast<int16_t>(std::min(T, v.n_vis - c * T));
+        k.diag = 0;
+        k.visual = 1;
+        P.kv.push_back(k);
+      }
+      for (int u = 0; u <= t; ++u) {
+        KvTile k{};
+        k.start = v.vis_start + v.n_vis + u * T;
+        k.len = static_cast<int16_t>(std::min(T, v.n_text - u * T));
+        k.diag = u == t;
+        k.visual = 0;
+        P.kv.push_back(k);
+      }
+      const int cnt = static_cast<int>(P.kv.size()) - kv_begin;
+      const int nsplit = (cnt + split_len - 1) / split_len;
+      for (int h : head_blocks) {
+        int part0 = -1;
+        if (nsplit > 1) {
+          part0 = P.n_parts;
+          P.n_parts += nsplit;
+          CombineGroup g{};
+          g.q_start = v.vis_start + v.n_vis + t * T;
+          g.q_len = std::min(T, v.n_text - t * T);
+          g.head = h;
+          g.part0 = part0;
+          g.nsplit = nsplit;
+          P.groups.push_back(g);
+        }
+        for (int s = 0; s < nsplit; ++s) {
+          // Even split of cnt tiles into nsplit chunks.
+          const int lo = static_cast<int>(static_cast<int64_t>(cnt) * s / nsplit);
+          const int hi = static_cast<int>(static_cast<int64_t>(cnt) * (s + 1) / nsplit);
+          WorkItem it{};
+          it.q_start = v.vis_start + v.n_vis + t * T;
+          it.q_len = std::min(T, v.n_text - t * T);
+          it.head = h;
+          it.kv_begin = kv_begin + lo;
+          it.kv_count = hi - lo;
+          it.part = nsplit > 1 ? part0 + s : -1;
+          it.video = b;
+          it.text_row0 = t * T;
+          items.push_back(it);
+        }
+      }
+    }
+  }
+  // Longest first; stable so that the heads of one row tile stay adjacent and
+  // share their K/V tiles through L2.
+  std::stable_sort(items.begin(), items.end(),
+                   [](const WorkItem& x, const WorkItem& y) { return x.kv_count > y.kv_count; });
+  P.items = std::move(items);
+
+  // Evidence column chunks.
+  for (int b = 0; b < a->num_videos; ++b)
+    for (int c = 0; c < P.videos[b].n_vis; c += 128) P.chunks.push_back(EvChunk{b, c});
+}
+
+}  // namespace
+
+struct evisel_ws {
+  int device = -1;
+  // device arena
+  void* arena = nullptr;
+  size_t arena_bytes = 0;
+  int* status = nullptr;
+  // pinned staging of the plan metadata
+  void* stage = nullptr;
+  size_t stage_bytes = 0;
+  cudaEvent_t stage_done = nullptr;
+  // current plan
+  std::vector<int32_t> key;
+  bool have_plan = false;
+  Plan plan;
+  WorkItem* d_items = nullptr;
+  KvTile* d_kv = nullptr;
+  VideoInfo* d_videos = nullptr;
+  CombineGroup* d_groups = nullptr;
+  EvChunk* d_chunks = nullptr;
+  float* d_part_o = nullptr;
+  float2* d_part_ml = nullptr;
+  float* d_spill = nullptr;
+  // last probe, for the evidence pass
+  bool probed = false;
+  const float* lse = nullptr;
+  int hq = 0;
+  int tokens_per_frame = 0;
+  cudaStream_t last_stream = nullptr;
+};
+
+namespace {
+
+std::vector<int32_t> plan_key(const evisel_probe_args* a) {
+  std::vector<int32_t> k = {a->num_videos, a->tokens_per_frame, a->hq, a->hkv, a->head_dim, a->tile};
+  for (int b = 0; b <= a->num_videos && a->num_videos > 0; ++b) k.push_back(a->cu_seqlens_h[b]);
+  for (int b = 0; b < a->num_videos; ++b) k.push_back(a->n_vis_h[b]);
+  int64_t rows = 0;
+  for (int b = 0; b < a->num_videos; ++b) rows += (a->n_vis_h[b] + a->tile - 1) / a->tile;
+  if (rows > 0) {
+    k.insert(k.end(), a->mask_row_ptr_h, a->mask_row_ptr_h + rows + 1);
+    k.insert(k.end(), a->mask_col_idx_h, a->mask_col_idx_h + a->mask_row_ptr_h[rows]);
+  }
+  return k;
+}
+
+template <typename T>
+size_t bytes_of(const std::vector<T>& v) { return v.size() * sizeof(T); }
+
+// Lays out the arena and uploads the plan metadata on `stream`.
+int install_plan(evisel_ws* ws, cudaStream_t stream) {
+  const Plan& P = ws->plan;
+  const int d = 128;   // partial rows are sized for the largest head_dim
+  size_t off = 0;
+  auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
+  const size_t o_items = take(bytes_of(P.items));
+  const size_t o_kv = take(bytes_of(P.kv));
+  const size_t o_videos = take(bytes_of(P.videos));
+  const size_t o_groups = take(bytes_of(P.groups));
+  const size_t o_chunks = take(bytes_of(P.chunks));
+  const size_t meta_bytes = off;
+  const size_t o_part_o = take(static_cast<size_t>(P.n_parts) * 128 * d * sizeof(float));
+  const size_t o_part_ml = take(static_cast<size_t>(P.n_parts) * 128 * sizeof(float2));
+  const size_t o_spill = take(static_cast<size_t>(P.spill_floats) * sizeof(float));
+  const size_t total = std::max<size_t>(off, 256);
+
+  if (total > ws->arena_bytes) {
+    if (ws->arena) {
+      cudaError_t e = cudaStreamSynchronize(stream);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+      cudaFree(ws->arena);
+      ws->arena = nullptr;
+      ws->arena_bytes = 0;
+    }
+    cudaError_t e = cudaMalloc(&ws->arena, total);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      return fail(EVISEL_ENOMEM, "workspace allocation of " + std::to_string(total) + " bytes failed");
+    }
+    ws->arena_bytes = total;
+  }
+  if (meta_bytes > ws->stage_bytes) {
+    if (ws->stage) {
+      cudaEventSynchronize(ws->stage_done);
+      cudaFreeHost(ws->stage);
+      ws->stage = nullptr;
+    }
+    if (cudaMallocHost(&ws->stage, meta_bytes) != cudaSuccess) {
+      cudaGetLastError();
+      ws->stage_bytes = 0;
+      return fail(EVISEL_ENOMEM, "pinned staging allocation failed");
+    }
+    ws->stage_bytes = meta_bytes;
+  }
+  // The staging buffer may still feed the previous upload.
+  cudaEventSynchronize(ws->stage_done);
+  char* h = static_cast<char*>(ws->stage);
+  if (!P.items.empty()) std::memcpy(h + o_items, P.items.data(), bytes_of(P.items));
+  if (!P.kv.empty()) std::memcpy(h + o_kv, P.kv.data(), bytes_of(P.kv));
+  if (!P.videos.empty()) std::memcpy(h + o_videos, P.videos.data(), bytes_of(P.videos));
+  if (!P.groups.empty()) std::memcpy(h + o_groups, P.groups.data(), bytes_of(P.groups));
+  if (!P.chunks.empty()) std::memcpy(h + o_chunks, P.chunks.data(), bytes_of(P.chunks));
+  char* base = static_cast<char*>(ws->arena);
+  if (meta_bytes > 0) {
+    cudaError_t e = cudaMemcpyAsync(base, h, meta_bytes, cudaMemcpyHostToDevice, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "plan upload");
+    e = cudaEventRecord(ws->stage_done, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+  }
+  ws->d_items = reinterpret_cast<WorkItem*>(base + o_items);
+  ws->d_kv = reinterpret_cast<KvTile*>(base + o_kv);
+  ws->d_videos = reinterpret_cast<VideoInfo*>(base + o_videos);
+  ws->d_groups = reinterpret_cast<CombineGroup*>(base + o_groups);
+  ws->d_chunks = reinterpret_cast<EvChunk*>(base + o_chunks);
+  ws->d_part_o = reinterpret_cast<float*>(base + o_part_o);
+  ws->d_part_ml = reinterpret_cast<float2*>(base + o_part_ml);
+  ws->d_spill = reinterpret_cast<float*>(base + o_spill);
+  return EVISEL_OK;
+}
+
+int create_ws(evisel_ws** out) {
+  evisel_ws* ws = new evisel_ws();
+  cudaError_t e = cudaGetDevice(&ws->device);
+  if (e == cudaSuccess) e = cudaMalloc(&ws->status, sizeof(int));
+  if (e == cudaSuccess) e = cudaMemset(ws->status, 0, sizeof(int));
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ws->stage_done, cudaEventDisableTiming);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    if (ws->status) cudaFree(ws->status);
+    delete ws;
+    return cuda_fail(e, "workspace creation");
+  }
+  *out = ws;
+  return EVISEL_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int evisel_probe_attention(const evisel_probe_args* args, void* stream_ptr, evisel_ws** ws_inout) {
+  g_last_error.clear();
+  if (!ws_inout) return fail(EVISEL_EINVAL, "ws_inout is NULL");
+  int rc = validate(args);
+  if (rc != EVISEL_OK) return rc;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
+  if (!*ws_inout) {
+    rc = create_ws(ws_inout);
+    if (rc != EVISEL_OK) return rc;
+  }
+  evisel_ws* ws = *ws_inout;
+  int dev = -1;
+  cudaGetDevice(&dev);
+  if (dev != ws->device) return fail(EVISEL_EINVAL, "workspace belongs to another device");
+
+  std::vector<int32_t> key = plan_key(args);
+  if (!ws->have_plan || key != ws->key) {
+    ws->plan = Plan();
+    build_plan(args, ws->plan);
+    ws->have_plan = false;
+    rc = install_plan(ws, stream);
+    if (rc != EVISEL_OK) return rc;
+    ws->key.swap(key);
+    ws->have_plan = true;
+  }
+  if (ws->last_stream != stream) {
+    // The plan metadata may have been uploaded on another stream.
+    cudaError_t e = cudaStreamWaitEvent(stream, ws->stage_done, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+  }
+  const Plan& P = ws->plan;
+  const float scale = args->softmax_scale > 0.f ? args->softmax_scale : 1.0f / std::sqrt(float(args->head_dim));
+
+  if (!P.items.empty()) {
+    ProbeLaunch L;
+    std::memset(&L, 0, sizeof(L));
+    rc = encode_map(&L.tm_q, args->q, P.n_tok, args->hq, args->head_dim, args->tile);
+    if (rc == EVISEL_OK) rc = encode_map(&L.tm_k, args->k, P.n_tok, args->hkv, args->head_dim, args->tile);
+    if (rc == EVISEL_OK) rc = encode_map(&L.tm_v, args->v, P.n_tok, args->hkv, args->head_dim, args->tile);
+    if (rc != EVISEL_OK) return rc;
+    L.items = ws->d_items;
+    L.kv = ws->d_kv;
+    L.videos = ws->d_videos;
+    L.o = args->o;
+    L.lse = args->lse;
+    L.spill = ws->d_spill;
+    L.part_o = ws->d_part_o;
+    L.part_ml = ws->d_part_ml;
+    L.status = ws->status;
+    L.n_items = static_cast<int>(P.items.size());
+    L.n_tok = P.n_tok;
+    L.hq = args->hq;
+    L.hkv = args->hkv;
+    L.head_dim = args->head_dim;
+    L.tile = args->tile;
+    L.scale = scale;
+    L.scale_log2 = scale * 1.4426950408889634f;
+    cudaError_t e = launch_probe_attn(L, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "probe_attn launch");
+    if (!P.groups.empty()) {
+      CombineLaunch C{};
+      C.groups = ws->d_groups;
+      C.part_o = ws->d_part_o;
+      C.part_ml = ws->d_part_ml;
+      C.o = args->o;
+      C.lse = args->lse;
+      C.n_groups = static_cast<int>(P.groups.size());
+      C.n_tok = P.n_tok;
+      C.hq = args->hq;
+      C.hkv = args->hkv;
+      C.head_dim = args->head_dim;
+      C.tile = args->tile;
+      e = launch_attn_combine(C, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "attn_combine launch");
+    }
+  }
+  ws->probed = true;
+  ws->lse = args->lse;
+  ws->hq = args->hq;
+  ws->tokens_per_frame = args->tokens_per_frame;
+  ws->last_stream = stream;
+  return EVISEL_OK;
+}
+
+int evisel_evidence_reduce(const evisel_ws* ws_c, float* tok, float* frame, float* head, float* aqf,
+                           int accumulate, void* stream_ptr) {
+  g_last_error.clear();
+  evisel_ws* ws = const_cast<evisel_ws*>(ws_c);
+  if (!ws) return fail(EVISEL_EINVAL, "workspace is NULL");
+  if (!ws->probed || !ws->have_plan) return fail(EVISEL_ESTATE, "no probe has run on this workspace");
+  const Plan& P = ws->plan;
+  if (P.videos.empty()) return EVISEL_OK;
+  if ((P.total_vis > 0 && (!tok || !frame)) || !head || (P.total_frames > 0 && !aqf))
+    return fail(EVISEL_EINVAL, "an output map is NULL");
+  if ((reinterpret_cast<uintptr_t>(tok) & 15u) != 0) return fail(EVISEL_EINVAL, "tok must be 16-byte aligned");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
+  EvidenceLaunch L{};
+  L.chunks = ws->d_chunks;
+  L.videos = ws->d_videos;
+  L.spill = ws->d_spill;
+  L.lse = ws->lse;
+  L.tok = tok;
+  L.frame = frame;
+  L.head = head;
+  L.aqf = aqf;
+  L.n_chunks = static_cast<int>(P.chunks.size());
+  L.n_videos = static_cast<int>(P.videos.size());
+  L.n_tok = P.n_tok;
+  L.hq = ws->hq;
+  L.tokens_per_frame = ws->tokens_per_frame;
+  L.total_vis = P.total_vis;
+  L.total_frames = P.total_frames;
+  L.accumulate = accumulate != 0;
+  cudaError_t e = launch_evidence(L, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "evidence launch");
+  ws->last_stream = stream;
+  return EVISEL_OK;
+}
+
+void evisel_free(evisel_ws* ws) {
+  if (!ws) return;
+  int prev = -1;
+  cudaGetDevice(&prev);
+  if (ws->device >= 0 && prev != ws->device) cudaSetDevice(ws->device);
+  cudaStreamSynchronize(ws->last_stream);
+  if (ws->stage_done) cudaEventSynchronize(ws->stage_done);
+  if (ws->arena) cudaFree(ws->arena);
+  if (ws->status) cudaFree(ws->status);
+  if (ws->stage) cudaFreeHost(ws->stage);
+  if (ws->stage_done) cudaEventDestroy(ws->stage_done);
+  if (prev >= 0 && prev != ws->device) cudaSetDevice(prev);
+  cudaGetLastError();
+  delete ws;
+}
+
+int evisel_status(evisel_ws* ws) {
+  g_last_error.clear();
+  if (!ws) return fail(EVISEL_EINVAL, "workspace is NULL");
+  cudaError_t e = cudaStreamSynchronize(ws->last_stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  int st = 0;
+  e = cudaMemcpy(&st, ws->status, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "status read");
+  if (st != 0) {
+    const int zero = 0;
+    cudaMemcpy(ws->status, &zero, sizeof(int), cudaMemcpyHostToDevice);
+  }
+  return st;
+}
+
+const char* evisel_strerror(int code) {
+  switch (code) {
+    case EVISEL_OK: return "success";
+    case EVISEL_EINVAL: return "invalid argument";
+    case EVISEL_EUNSUPPORTED: return "unsupported shape or parameter";
+    case EVISEL_EMASK: return "invalid block mask";
+    case EVISEL_ECUDA: return "CUDA error";
+    case EVISEL_ENOMEM: return "out of memory";
+    case EVISEL_ETIMEOUT: return "device wait timed out";
+    case EVISEL_EBOUNDS: return "device index check failed";
+    case EVISEL_ESTATE: return "no probe has run on this workspace";
+    default: return "unknown status";
+  }
+}
+
+const char* evisel_last_error(void) { return g_last_error.c_str(); }
+
+int64_t evisel_workspace_bytes(const evisel_ws* ws) {
+  return ws ? static_cast<int64_t>(ws->arena_bytes) : 0;
+}
+
+}  // extern "C"

@@ -1,0 +1,122 @@
+// Internal structures shared by the host planner (evisel_capi.cpp) and the
+// sm_103a kernels. Not part of the public ABI.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace evisel {
+
+// One kept kv tile of a work item: keys [start, start + len) (global token
+// indices, one video). `diag` marks the tile that holds the query tile's own
+// positions: causal masking inside it. `visual` marks visual-token tiles, whose
+// logits the text rows spill for the evidence pass.
+struct KvTile {
+  int32_t start;
+  int16_t len;
+  uint8_t diag;
+  uint8_t visual;
+};
+static_assert(sizeof(KvTile) == 8, "KvTile is packed into 8 bytes");
+
+// One CTA's work: a query row tile of one (or, for 64-token tiles, two
+// consecutive) query heads against a contiguous range of its kept kv tiles.
+struct WorkItem {
+  int32_t q_start;    // global index of the tile's first query token
+  int32_t q_len;      // valid rows (<= tile)
+  int32_t head;       // first query head
+  int32_t kv_begin;   // index into the KvTile list
+  int32_t kv_count;   // >= 1
+  int32_t part;       // split-KV partial slot, -1 when the item writes O/LSE itself
+  int32_t video;      // video index
+  int32_t text_row0;  // index of the first row among the video's text rows, -1 for visual rows
+};
+static_assert(sizeof(WorkItem) == 32, "WorkItem is 32 bytes");
+
+// Per-video layout used by the spill and the evidence pass.
+struct VideoInfo {
+  int64_t spill_off;  // float offset of this video's [hq, n_text, vis_pitch] logit block
+  int32_t vis_start;  // global index of its first visual token
+  int32_t n_vis;
+  int32_t n_text;
+  int32_t vis_pitch;  // n_vis rounded up to a multiple of 4 (row pitch of the spill)
+  int32_t vis_off;    // column offset of its tokens in the token map
+  int32_t frame_off;  // column offset of its frames in the frame map
+};
+static_assert(sizeof(VideoInfo) == 32, "VideoInfo is 32 bytes");
+
+// A text row tile whose kv range was split over several items: the partials
+// in slots [part0, part0 + nsplit) are merged by the combine kernel.
+struct CombineGroup {
+  int32_t q_start;
+  int32_t q_len;
+  int32_t head;
+  int32_t part0;
+  int32_t nsplit;
+  int32_t pad0, pad1, pad2;
+};
+static_assert(sizeof(CombineGroup) == 32, "CombineGroup is 32 bytes");
+
+// Column chunk of the evidence pass: 128 visual tokens of one video.
+struct EvChunk {
+  int32_t video;
+  int32_t col0;       // first visual column within the video
+};
+
+struct ProbeLaunch {
+  CUtensorMap tm_q, tm_k, tm_v;     // 3-D maps {d, heads, tokens}, box {64, 1, tile}, 128B swizzle
+  const WorkItem* items;
+  const KvTile* kv;
+  const VideoInfo* videos;
+  void* o;                          // bf16 [N, hq, d]
+  float* lse;                       // [hq, N]
+  float* spill;                     // text-row logits
+  float* part_o;                    // [slots, 128, d] fp32, unnormalised
+  float2* part_ml;                  // [slots, 128] (running max in log2 units, row sum)
+  int* status;                      // device status word
+  int n_items;
+  int n_tok;
+  int hq, hkv, head_dim, tile;
+  float scale_log2;                 // softmax_scale * log2(e)
+  float scale;                      // softmax_scale
+};
+
+struct CombineLaunch {
+  const CombineGroup* groups;
+  const float* part_o;
+  const float2* part_ml;
+  void* o;
+  float* lse;
+  int n_groups;
+  int n_tok, hq, hkv, head_dim, tile;
+};
+
+struct EvidenceLaunch {
+  const EvChunk* chunks;
+  const VideoInfo* videos;
+  const float* spill;
+  const float* lse;
+  float* tok;
+  float* frame;
+  float* head;
+  float* aqf;
+  int n_chunks;
+  int n_videos;
+  int n_tok, hq, tokens_per_frame;
+  int total_vis, total_frames;
+  int accumulate;
+};
+
+// Kernel launchers (defined in the .cu files).
+cudaError_t launch_probe_attn(const ProbeLaunch& L, cudaStream_t stream);
+cudaError_t launch_attn_combine(const CombineLaunch& L, cudaStream_t stream);
+cudaError_t launch_evidence(const EvidenceLaunch& L, cudaStream_t stream);
+
+// Bounded waits give up after this many nanoseconds of %globaltimer.
+constexpr uint64_t kWaitTimeoutNs = 2000000000ull;
+
+constexpr int kStatusTimeout = -6;   // == EVISEL_ETIMEOUT
+constexpr int kStatusBounds = -7;    // == EVISEL_EBOUNDS
+
+}  // namespace evisel

@@ -39,16 +39,20 @@ __all__ = [
 ]
 
 
-def bf16_round(x: np.ndarray) -> np.ndarray:
+def bf16_round(x: np.ndarray, inplace: bool = False) -> np.ndarray:
     """Round float32 values to the nearest bfloat16 (ties to even); returns float32."""
-    x = np.array(x, dtype=np.float32, copy=True, order="C")
+    if not (inplace and x.dtype == np.float32 and x.flags.c_contiguous):
+        x = np.array(x, dtype=np.float32, copy=True, order="C")
     flat = x.reshape(-1).view(np.uint32)
-    step = 1 << 22
-    for a in range(0, flat.size, step):        # finite inputs only: no uint32 overflow
+    step = 1 << 18                              # cache-sized chunks, finite inputs (no uint32 overflow)
+    lsb = np.empty(step, np.uint32)
+    for a in range(0, flat.size, step):
         u = flat[a:a + step]
-        lsb = (u >> 16) & np.uint32(1)
-        u += np.uint32(0x7FFF)
-        u += lsb
+        r = lsb[:u.size]
+        np.right_shift(u, 16, out=r)
+        np.bitwise_and(r, 1, out=r)
+        r += np.uint32(0x7FFF)
+        u += r
         u &= np.uint32(0xFFFF0000)
     return x
 
@@ -194,9 +198,11 @@ def make_probe(cfg: ProbeConfig, layer: int = 0, mask=None) -> Probe:
     rng = np.random.default_rng(seed)
     n, d = cfg.n_tot, cfg.head_dim
     div = np.float32(math.sqrt(d)) if cfg.scale_inputs else np.float32(1.0)
-    q = rng.standard_normal((n, cfg.hq, d), dtype=np.float32) / div
-    k = rng.standard_normal((n, cfg.hkv, d), dtype=np.float32) / div
-    v = rng.standard_normal((n, cfg.hkv, d), dtype=np.float32) / div
+    q = rng.standard_normal((n, cfg.hq, d), dtype=np.float32)
+    k = rng.standard_normal((n, cfg.hkv, d), dtype=np.float32)
+    v = rng.standard_normal((n, cfg.hkv, d), dtype=np.float32)
+    for x in (q, k, v):
+        np.divide(x, div, out=x)
     cu = np.zeros(cfg.num_videos + 1, dtype=np.int64)
     cu[1:] = np.cumsum(cfg.seqlens)
     planted = _planted_frames(cfg)
@@ -215,6 +221,6 @@ def make_probe(cfg: ProbeConfig, layer: int = 0, mask=None) -> Probe:
     if mask is None:
         mask = build_mask(cfg)
     row_ptr, col_idx = mask
-    return Probe(cfg, layer, bf16_round(q), bf16_round(k), bf16_round(v),
+    return Probe(cfg, layer, bf16_round(q, True), bf16_round(k, True), bf16_round(v, True),
                  cu.astype(np.int32), np.asarray(cfg.n_vis, dtype=np.int32),
                  row_ptr, col_idx, planted)
