@@ -136,6 +136,41 @@ const char* evisel_last_error(void);
 /* Bytes of device memory currently held by the workspace (0 for NULL). */
 int64_t evisel_workspace_bytes(const evisel_ws* ws);
 
+/* ---- Entry point that allocates nothing ---------------------------------------
+ * The paper has no counterpart to this call. It serves callers of this library
+ * that cannot call cudaMalloc on their serving path: servers that hand all device
+ * memory to their own pool up front, real-time paths where an allocation (and the
+ * device synchronisation that cudaFree implies) is not acceptable, or hosts that
+ * forbid the library any allocator use of its own.
+ *
+ * It computes exactly what evisel_probe_attention() followed by
+ * evisel_evidence_reduce() compute, with the same arguments and outputs (O and
+ * LSE through `args`, the four evidence maps through tok/frame/head/aqf), but it
+ * allocates nothing: no cudaMalloc, cudaFree, pinned memory or workspace. All of
+ * its scratch -- the work plan, the split-KV partials of the text rows and the
+ * text-row logit spill -- lives in one static device array of
+ * EVISEL_NOALLOC_SCRATCH_BYTES (64 MiB), which every GPU that loads this library
+ * holds until the process exits.
+ *   - Limit: a problem whose scratch does not fit is rejected with EVISEL_ENOMEM
+ *     (evisel_last_error() states the bytes needed) before anything is enqueued.
+ *     The spill dominates: about hq * n_text * n_vis * 4 bytes per video, e.g.
+ *     28 heads x 64 text x 4096 visual tokens = 29 MiB fits; the 65,664-token
+ *     probe (940 MiB) does not -- use evisel_probe_attention() for it.
+ *   - Set-up: the first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current) and caches it; make that
+ *     first call before any stream capture begins.
+ *   - Sharing: all calls use the same array, which keeps the previous call's
+ *     contents; each call clears what must start at zero (the device status
+ *     word). Calls whose GPU work overlaps (different streams, or host threads
+ *     without ordering) race on the array: order them on one stream.
+ *   - device_status: NULL -> the call is asynchronous on `stream`; otherwise it
+ *     waits for `stream` and stores the device status word there (EVISEL_OK or
+ *     EVISEL_ETIMEOUT).
+ * Errors: as evisel_probe_attention() and evisel_evidence_reduce(). */
+#define EVISEL_NOALLOC_SCRATCH_BYTES (64LL << 20)
+int evisel_probe_evidence_noalloc(const evisel_probe_args* args, float* tok, float* frame, float* head,
+                                  float* aqf, int accumulate, void* stream, int* device_status);
+
 #ifdef __cplusplus
 }
 #endif

@@ -76,6 +76,9 @@ def load(path: str = LIB_PATH):
     lib.evisel_last_error.restype = ctypes.c_char_p
     lib.evisel_workspace_bytes.argtypes = [vp]
     lib.evisel_workspace_bytes.restype = ctypes.c_int64
+    lib.evisel_probe_evidence_noalloc.argtypes = [ctypes.POINTER(ProbeArgs), vp, vp, vp, vp, i32, vp,
+                                                  ctypes.POINTER(ctypes.c_int)]
+    lib.evisel_probe_evidence_noalloc.restype = i32
     _lib = lib
     return lib
 
@@ -197,3 +200,28 @@ def evisel_status(ws):
 
 def evisel_free(ws):
     ws.free()
+
+
+NOALLOC_SCRATCH_BYTES = 64 << 20
+
+
+def evisel_probe_evidence_noalloc(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
+                                  tok, frame, head, aqf, accumulate=False, softmax_scale=0.0, stream=None,
+                                  wait_status=True):
+    """Probe + evidence through the entry point that allocates nothing.
+
+    For callers that cannot let the library call cudaMalloc: every output
+    (o, lse and the four maps) is passed in, and the library's scratch is a
+    fixed 64 MiB static device array (problems that need more are rejected).
+    Returns the device status word when ``wait_status`` (the call then waits
+    for the stream), else None.
+    """
+    lib = load()
+    args, keep = make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
+                           softmax_scale)
+    status = ctypes.c_int(0)
+    _check(lib.evisel_probe_evidence_noalloc(ctypes.byref(args), tok.data_ptr(), frame.data_ptr(), head.data_ptr(),
+                                             aqf.data_ptr(), int(bool(accumulate)), _stream_handle(stream),
+                                             ctypes.byref(status) if wait_status else None))
+    del keep
+    return int(status.value) if wait_status else None

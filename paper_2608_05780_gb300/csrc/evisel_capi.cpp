@@ -275,6 +275,16 @@ void build_plan(const evisel_probe_args* a, Plan& P) {
 
 }  // namespace
 
+// Helpers shared with the other host entry points of the library.
+namespace evisel {
+int validate_probe_args(const evisel_probe_args* a) { return validate(a); }
+int encode_tensor_map(CUtensorMap* map, const void* base, int n_tok, int heads, int d, int rows) {
+  return encode_map(map, base, n_tok, heads, d, rows);
+}
+int set_last_error(int code, const char* msg) { return fail(code, msg); }
+void clear_last_error() { g_last_error.clear(); }
+}  // namespace evisel
+
 struct evisel_ws {
   int device = -1;
   // device arena

@@ -113,6 +113,11 @@ cudaError_t launch_probe_attn(const ProbeLaunch& L, cudaStream_t stream);
 cudaError_t launch_attn_combine(const CombineLaunch& L, cudaStream_t stream);
 cudaError_t launch_evidence(const EvidenceLaunch& L, cudaStream_t stream);
 
+// Host helpers defined in evisel_capi.cpp.
+int encode_tensor_map(CUtensorMap* map, const void* base, int n_tok, int heads, int d, int rows);
+int set_last_error(int code, const char* msg);
+void clear_last_error();
+
 // Bounded waits give up after this many nanoseconds of %globaltimer.
 constexpr uint64_t kWaitTimeoutNs = 2000000000ull;
 
