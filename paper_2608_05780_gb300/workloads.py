@@ -124,6 +124,11 @@ CONFIGS = {
         plant=_plant_count(0.02, (1024,)), seed=3, mask_seed=3,
         description="1024 frames x 64 tokens + 128 text (65,664 tokens); 28q/4kv, d=128; "
                     "sink+16-window+32 random tiles per visual row tile"),
+    "prof24k": ProbeConfig(
+        "prof24k", (384,), 64, (128,), 28, 4, 128, 128, 16, extra=32,
+        plant=_plant_count(0.02, (384,)), seed=3, mask_seed=3,
+        description="profiling-size variant of long65k: 384 frames x 64 tokens + 128 text (24,704 tokens); "
+                    "same heads, tiles and mask recipe; inputs still larger than L2"),
     "varlen8": ProbeConfig(
         "varlen8", _C5_FRAMES, 16, _C5_TEXT, 28, 4, 128, 128, 8,
         plant=_plant_count(0.05, _C5_FRAMES), seed=4, qkv_seed=(4, 1),
