@@ -40,12 +40,13 @@ __global__ void attn_combine_kernel(const __grid_constant__ CombineLaunch L) {
   const int qpos = g.q_start + row_local;
 
   float mmax = -INFINITY;
-  for (int s = 0; s < g.nsplit; ++s) mmax = fmaxf(mmax, L.part_ml[(int64_t)(g.part0 + s) * kRows + row].x);
+  for (int s = 0; s < g.nsplit; ++s)
+    mmax = fmaxf(mmax, L.part_ml[(g.part0 + static_cast<int64_t>(s) * g.stride) * kRows + row].x);
   const float msafe = mmax == -INFINITY ? 0.f : mmax;
   float lsum = 0.f;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   for (int s = 0; s < g.nsplit; ++s) {
-    const int64_t slot = g.part0 + s;
+    const int64_t slot = g.part0 + static_cast<int64_t>(s) * g.stride;
     const float2 ml = L.part_ml[slot * kRows + row];
     const float w = exp2f(ml.x - msafe);
     lsum += w * ml.y;

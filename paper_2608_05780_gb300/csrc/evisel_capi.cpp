@@ -140,13 +140,13 @@ int validate(const evisel_probe_args* a) {
 void build_plan(const evisel_probe_args* a, Plan& P) {
   const int T = a->tile;
   const int hq = a->hq, gq = a->hq / a->hkv;
-  const int hp = 128 / T;                      // heads per CTA
+  const int hp = 128 / T;                      // heads per slot
   P.n_tok = a->num_videos ? a->cu_seqlens_h[a->num_videos] : 0;
 
-  // Head blocks: consecutive heads of one KV group.
+  // Head blocks: up to kSlots * hp consecutive heads of one KV group.
   std::vector<int> head_blocks;
   for (int g = 0; g < a->hkv; ++g)
-    for (int hh = 0; hh < gq; hh += hp) head_blocks.push_back(g * gq + hh);
+    for (int hh = 0; hh < gq; hh += kSlots * hp) head_blocks.push_back(g * gq + hh);
 
   // Videos.
   int64_t spill = 0;
@@ -234,15 +234,20 @@ void build_plan(const evisel_probe_args* a, Plan& P) {
       for (int h : head_blocks) {
         int part0 = -1;
         if (nsplit > 1) {
+          // kSlots partial slots per split, interleaved: split k of slot s
+          // sits in part0 + k * kSlots + s.
           part0 = P.n_parts;
-          P.n_parts += nsplit;
-          CombineGroup g{};
-          g.q_start = v.vis_start + v.n_vis + t * T;
-          g.q_len = std::min(T, v.n_text - t * T);
-          g.head = h;
-          g.part0 = part0;
-          g.nsplit = nsplit;
-          P.groups.push_back(g);
+          P.n_parts += kSlots * nsplit;
+          for (int slot = 0; slot < kSlots && (h % gq) + slot * hp < gq; ++slot) {
+            CombineGroup g{};
+            g.q_start = v.vis_start + v.n_vis + t * T;
+            g.q_len = std::min(T, v.n_text - t * T);
+            g.head = h + slot * hp;
+            g.part0 = part0 + slot;
+            g.nsplit = nsplit;
+            g.stride = kSlots;
+            P.groups.push_back(g);
+          }
         }
         for (int s = 0; s < nsplit; ++s) {
           // Even split of cnt tiles into nsplit chunks.
@@ -254,7 +259,7 @@ void build_plan(const evisel_probe_args* a, Plan& P) {
           it.head = h;
           it.kv_begin = kv_begin + lo;
           it.kv_count = hi - lo;
-          it.part = nsplit > 1 ? part0 + s : -1;
+          it.part = nsplit > 1 ? part0 + kSlots * s : -1;
           it.video = b;
           it.text_row0 = t * T;
           items.push_back(it);

@@ -20,15 +20,21 @@ struct KvTile {
 };
 static_assert(sizeof(KvTile) == 8, "KvTile is packed into 8 bytes");
 
-// One CTA's work: a query row tile of one (or, for 64-token tiles, two
-// consecutive) query heads against a contiguous range of its kept kv tiles.
+// Query-head slots per work item. A slot is one 128-row MMA tile: one head
+// for 128-token tiles, two consecutive heads for 64-token tiles. Both slots of
+// an item belong to one KV group and share every K/V tile the CTA loads.
+constexpr int kSlots = 2;
+
+// One CTA's work: a query row tile of up to kSlots * (128 / tile) consecutive
+// query heads of one KV group against a contiguous range of its kept kv tiles.
+// Heads past the end of the group are left out.
 struct WorkItem {
   int32_t q_start;    // global index of the tile's first query token
   int32_t q_len;      // valid rows (<= tile)
   int32_t head;       // first query head
   int32_t kv_begin;   // index into the KvTile list
   int32_t kv_count;   // >= 1
-  int32_t part;       // split-KV partial slot, -1 when the item writes O/LSE itself
+  int32_t part;       // split-KV partial of slot 0 (slot s uses part + s), -1 when the item writes O/LSE
   int32_t video;      // video index
   int32_t text_row0;  // index of the first row among the video's text rows, -1 for visual rows
 };
@@ -46,15 +52,16 @@ struct VideoInfo {
 };
 static_assert(sizeof(VideoInfo) == 32, "VideoInfo is 32 bytes");
 
-// A text row tile whose kv range was split over several items: the partials
-// in slots [part0, part0 + nsplit) are merged by the combine kernel.
+// One slot of a text row tile whose kv range was split over several items:
+// the partial of split k sits in partial slot part0 + k * stride.
 struct CombineGroup {
   int32_t q_start;
   int32_t q_len;
   int32_t head;
   int32_t part0;
   int32_t nsplit;
-  int32_t pad0, pad1, pad2;
+  int32_t stride;
+  int32_t pad1, pad2;
 };
 static_assert(sizeof(CombineGroup) == 32, "CombineGroup is 32 bytes");
 

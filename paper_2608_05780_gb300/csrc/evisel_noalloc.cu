@@ -111,7 +111,7 @@ void make_plan(const evisel_probe_args* a, Counts& c, const Out* o) {
       const int cnt = static_cast<int>(c.kv) - kv_begin;
       max_visual = std::max(max_visual, cnt);
       for (int g = 0; g < a->hkv; ++g)
-        for (int hh = 0; hh < gq; hh += hp, ++c.items)
+        for (int hh = 0; hh < gq; hh += kSlots * hp, ++c.items)
           if (o) o->items[c.items] = WorkItem{v.vis_start + t * T, std::min(T, v.n_vis - t * T), g * gq + hh,
                                               kv_begin, cnt, -1, b, -1};
     }
@@ -133,20 +133,20 @@ void make_plan(const evisel_probe_args* a, Counts& c, const Out* o) {
       const int q_start = v.vis_start + v.n_vis + t * T;
       const int q_len = std::min(T, v.n_text - t * T);
       for (int g = 0; g < a->hkv; ++g) {
-        for (int hh = 0; hh < gq; hh += hp) {
+        for (int hh = 0; hh < gq; hh += kSlots * hp) {
           const int h = g * gq + hh;
           int part0 = -1;
           if (nsplit > 1) {
             part0 = static_cast<int>(c.parts);
-            c.parts += nsplit;
-            if (o) o->groups[c.groups] = CombineGroup{q_start, q_len, h, part0, nsplit, 0, 0, 0};
-            ++c.groups;
+            c.parts += kSlots * nsplit;
+            for (int slot = 0; slot < kSlots && hh + slot * hp < gq; ++slot, ++c.groups)
+              if (o) o->groups[c.groups] = CombineGroup{q_start, q_len, h + slot * hp, part0 + slot, nsplit, kSlots, 0, 0};
           }
           for (int s = 0; s < nsplit; ++s, ++c.items) {
             const int lo = static_cast<int>(static_cast<int64_t>(cnt) * s / nsplit);
             const int hi = static_cast<int>(static_cast<int64_t>(cnt) * (s + 1) / nsplit);
             if (o) o->items[c.items] = WorkItem{q_start, q_len, h, kv_begin + lo, hi - lo,
-                                                nsplit > 1 ? part0 + s : -1, b, t * T};
+                                                nsplit > 1 ? part0 + kSlots * s : -1, b, t * T};
           }
         }
       }

@@ -2,14 +2,24 @@
 // (the paper's sparse probe, Sec. 3.2 Eq. 1, with exact token logits on every
 // kept tile: Appendix Eq. 8 in token form and the row normalisation of Eq. 11).
 //
-// One CTA computes one work item: a 128-row query tile (one head for 128-token
-// tiles, two heads of one KV group for 64-token tiles) against a list of kept
-// kv tiles. Warp roles:
-//   warps 0-3  softmax + epilogue, one thread per query row (= TMEM lane)
-//   warp 4     TMA producer: Q once, then K_j / V_j into an NS-deep smem ring
-//   warp 5     MMA issuer (one thread): S_j = Q K_j^T into a double-buffered
-//              TMEM S, O += P_j V_j with P_j read from TMEM (bf16)
-// TMEM columns: S0 | S1 | P0 | P1 | O.
+// One CTA computes one work item: a query row tile against a list of kept kv
+// tiles for two "slots" of query heads of one KV group. A slot is one 128-row
+// MMA tile (one head for 128-token tiles, two heads for 64-token tiles); both
+// slots use every K/V tile the CTA loads, and each slot's softmax runs while
+// the tensor core works on the other slot.
+//
+// Warp roles (320 threads):
+//   warps 0-3  softmax + epilogue of slot 0, one thread per query row (TMEM lane)
+//   warps 4-7  softmax + epilogue of slot 1
+//   warp 8     TMA producer: Q of both slots, then K_j / V_j into NS-deep rings
+//   warp 9     MMA issuer; the warp walks the tiles together and one elected
+//              lane issues, per kv tile j:
+//                O0 += P0_j V_j,  S0_{j+1} = Q0 K_{j+1}^T,
+//                O1 += P1_j V_j,  S1_{j+1} = Q1 K_{j+1}^T
+// TMEM columns per slot: S (TILE) | O (D). P_j (bf16) is written over the
+// first half of its own S_j columns and read from there by the P.V MMA; the
+// slot's next S is issued after that P.V, and the tcgen05 MMAs of one thread
+// execute in issue order.
 // Online softmax in fp32 (log2 domain) with lazy rescaling: the running max is
 // only moved when it grows by more than 2^8, so O in TMEM is rescaled rarely.
 // Text row tiles also spill their logits onto visual keys for the evidence
@@ -24,47 +34,50 @@
 namespace evisel {
 namespace {
 
-constexpr int kThreads = 192;
+static_assert(kSlots == 2, "the kernel runs two slots per work item");
+constexpr int kThreads = 320;
+constexpr int kWarpProducer = 8;
+constexpr int kWarpMma = 9;
 constexpr int kRows = 128;
 constexpr float kRescaleThreshold = 8.0f;   // log2 units
 constexpr float kLn2 = 0.69314718055994531f;
 
 template <int TILE, int D, int NS>
 struct Cfg {
-  static constexpr int HP = kRows / TILE;        // query heads per CTA
+  static constexpr int HP = kRows / TILE;        // query heads per slot
   static constexpr int KB = D / 64;              // 128-byte swizzle column blocks along d
-  static constexpr int Q_BYTES = kRows * D * 2;
-  static constexpr int Q_BLOCK = kRows * 128;    // one column block of Q
+  static constexpr int Q_BYTES = kRows * D * 2;  // one slot
+  static constexpr int Q_BLOCK = kRows * 128;    // one column block of a slot's Q
   static constexpr int KV_BLOCK = TILE * 128;    // one column block of a K/V tile
   static constexpr int KV_BYTES = TILE * D * 2;
-  static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = OFF_Q + Q_BYTES;
+  static constexpr int OFF_Q = 0;                        // two slots
+  static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;
   static constexpr int OFF_V = OFF_K + NS * KV_BYTES;
   static constexpr int OFF_BAR = OFF_V + NS * KV_BYTES;
   // barrier indices
   static constexpr int B_Q = 0;
-  static constexpr int B_KF = 1;
-  static constexpr int B_KE = B_KF + NS;
-  static constexpr int B_VF = B_KE + NS;
-  static constexpr int B_VE = B_VF + NS;
-  static constexpr int B_SF = B_VE + NS;   // 2
-  static constexpr int B_PF = B_SF + 2;    // 2
-  static constexpr int B_PV = B_PF + 2;    // 2
-  static constexpr int B_OF = B_PV + 2;
-  static constexpr int B_DRAIN = B_OF + 1;
+  static constexpr int B_KF = 1;             // NS: K tile landed
+  static constexpr int B_KE = B_KF + NS;     // NS: K tile consumed by both S MMAs
+  static constexpr int B_VF = B_KE + NS;     // NS: V tile landed
+  static constexpr int B_VE = B_VF + NS;     // NS: V tile consumed by both P.V MMAs
+  static constexpr int B_SF = B_VE + NS;     // 2 (per slot): S_j computed
+  static constexpr int B_PF = B_SF + 2;      // 2 (per slot): P_j written (128 arrivals)
+  static constexpr int B_OF = B_PF + 2;      // 2 (per slot): O complete
+  static constexpr int B_DRAIN = B_OF + 2;
   static constexpr int N_BARS = B_DRAIN + 1;
   static constexpr int OFF_MISC = OFF_BAR + N_BARS * 8;
   static constexpr int SMEM_USED = OFF_MISC + 16;
-  // TMEM columns (32-bit)
-  static constexpr int COL_S0 = 0;
-  static constexpr int COL_P0 = 2 * TILE;
-  static constexpr int COL_O = 3 * TILE;
-  static constexpr int TMEM_COLS = (3 * TILE + D <= 256) ? 256 : 512;
+  // TMEM columns (32-bit): slot s occupies [s * SLOT_COLS, (s + 1) * SLOT_COLS)
+  static constexpr int SLOT_COLS = TILE + D;
+  static constexpr int COL_S = 0;
+  static constexpr int COL_O = TILE;
+  static constexpr int TMEM_COLS = (2 * SLOT_COLS <= 256) ? 256 : 512;
   // Dynamic smem requested: enough to keep TMEM demand per SM within 512 columns.
   static constexpr int SMEM_MIN = TMEM_COLS == 512 ? 117 * 1024 : 78 * 1024;
   static constexpr int SMEM_BYTES = (SMEM_USED + 1024 > SMEM_MIN) ? SMEM_USED + 1024 : SMEM_MIN;
   static_assert(SMEM_USED + 1024 <= 232448, "shared memory budget");
   static_assert((OFF_K % 1024) == 0 && (OFF_V % 1024) == 0 && (KV_BYTES % 1024) == 0, "1 KB aligned tiles");
+  static_assert(2 * SLOT_COLS <= 512, "TMEM budget");
 };
 
 __device__ __forceinline__ void record_failure(volatile int* abort_flag, int* status, int code) {
@@ -73,60 +86,83 @@ __device__ __forceinline__ void record_failure(volatile int* abort_flag, int* st
 }
 
 // Bounded wait whose outcome is uniform across the warp, so that the warp stays
-// converged for the warp-collective tcgen05.ld / tcgen05.st that follow.
+// converged for the warp-collective tcgen05 operations that follow.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
   const bool ok = ptx::mbar_wait(bar, parity, abort_flag, kWaitTimeoutNs);
   return __all_sync(0xffffffffu, ok);
 }
 
+// Heads of the item's KV group from its first head on.
+__device__ __forceinline__ int heads_left(const ProbeLaunch& L, int head) {
+  const int gq = L.hq / L.hkv;
+  return gq - head % gq;
+}
+
 template <int TILE, int D, int NS>
-__device__ __forceinline__ void producer(const ProbeLaunch& L, const WorkItem& it, uint32_t sbase,
+__device__ __forceinline__ void producer(const ProbeLaunch& L, const WorkItem& it, uint32_t sbase_in,
                                          volatile int* abort_flag) {
   using C = Cfg<TILE, D, NS>;
+  const uint32_t sbase = __shfl_sync(0xffffffffu, sbase_in, 0);
   auto bar = [&](int i) { return sbase + C::OFF_BAR + 8u * i; };
-  const int gq = L.hq / L.hkv;
-  const int g = it.head / gq;
-  const bool second_ok = (C::HP == 1) || ((it.head + 1) < L.hq && (it.head + 1) / gq == g);
+  const int head0 = __shfl_sync(0xffffffffu, it.head, 0);
+  const int q_start = __shfl_sync(0xffffffffu, it.q_start, 0);
+  const int n = __shfl_sync(0xffffffffu, it.kv_count, 0);
+  const int kv_begin = __shfl_sync(0xffffffffu, it.kv_begin, 0);
+  const int g = head0 / (L.hq / L.hkv);
+  const int left = heads_left(L, head0);
+  const int nslots = left > C::HP ? 2 : 1;
   const uint64_t pol_q = ptx::l2_policy_evict_first();
   const uint64_t pol_kv = ptx::l2_policy_evict_last();
-  ptx::tma_prefetch_desc(&L.tm_q);
-  ptx::tma_prefetch_desc(&L.tm_k);
-  ptx::tma_prefetch_desc(&L.tm_v);
-
-  ptx::mbar_arrive_expect_tx(bar(C::B_Q), C::Q_BYTES);
+  uint32_t leader = 0;
+  if (ptx::elect_one(leader)) {
+    ptx::tma_prefetch_desc(&L.tm_q);
+    ptx::tma_prefetch_desc(&L.tm_k);
+    ptx::tma_prefetch_desc(&L.tm_v);
+    ptx::mbar_arrive_expect_tx(bar(C::B_Q), nslots * C::Q_BYTES);
+    for (int slot = 0; slot < nslots; ++slot) {
 #pragma unroll
-  for (int hp = 0; hp < C::HP; ++hp) {
-    const int h = (hp == 0 || second_ok) ? it.head + hp : it.head;
+      for (int hp = 0; hp < C::HP; ++hp) {
+        // A head past the group's end loads the first head again; its rows are never stored.
+        const int h = slot * C::HP + hp < left ? head0 + slot * C::HP + hp : head0;
 #pragma unroll
-    for (int kb = 0; kb < C::KB; ++kb)
-      ptx::tma_load_3d(sbase + C::OFF_Q + kb * C::Q_BLOCK + hp * TILE * 128, &L.tm_q, bar(C::B_Q), kb * 64, h,
-                       it.q_start, pol_q);
+        for (int kb = 0; kb < C::KB; ++kb)
+          ptx::tma_load_3d(sbase + C::OFF_Q + slot * C::Q_BYTES + kb * C::Q_BLOCK + hp * TILE * 128, &L.tm_q,
+                           bar(C::B_Q), kb * 64, h, q_start, pol_q);
+      }
+    }
   }
+  __syncwarp();
 
   int k_issued = 0, v_issued = 0;
-  for (int j = 0; j < it.kv_count; ++j) {
+  for (int j = 0; j < n; ++j) {
     const int s = j % NS;
     const int u = j / NS;
-    const KvTile kv = L.kv[it.kv_begin + j];
-    if (u > 0 && !ptx::mbar_wait(bar(C::B_KE + s), (u - 1) & 1, abort_flag, kWaitTimeoutNs)) {
-      record_failure(abort_flag, L.status, kStatusTimeout);
+    const int kv_start = __shfl_sync(0xffffffffu, L.kv[kv_begin + j].start, 0);
+    if (u > 0 && !warp_wait(bar(C::B_KE + s), (u - 1) & 1, abort_flag)) {
+      if ((threadIdx.x & 31) == leader) record_failure(abort_flag, L.status, kStatusTimeout);
       break;
     }
-    ptx::mbar_arrive_expect_tx(bar(C::B_KF + s), C::KV_BYTES);
+    if (ptx::elect_one(leader)) {
+      ptx::mbar_arrive_expect_tx(bar(C::B_KF + s), C::KV_BYTES);
 #pragma unroll
-    for (int kb = 0; kb < C::KB; ++kb)
-      ptx::tma_load_3d(sbase + C::OFF_K + s * C::KV_BYTES + kb * C::KV_BLOCK, &L.tm_k, bar(C::B_KF + s), kb * 64,
-                       g, kv.start, pol_kv);
+      for (int kb = 0; kb < C::KB; ++kb)
+        ptx::tma_load_3d(sbase + C::OFF_K + s * C::KV_BYTES + kb * C::KV_BLOCK, &L.tm_k, bar(C::B_KF + s), kb * 64,
+                         g, kv_start, pol_kv);
+    }
+    __syncwarp();
     k_issued = j + 1;
-    if (u > 0 && !ptx::mbar_wait(bar(C::B_VE + s), (u - 1) & 1, abort_flag, kWaitTimeoutNs)) {
-      record_failure(abort_flag, L.status, kStatusTimeout);
+    if (u > 0 && !warp_wait(bar(C::B_VE + s), (u - 1) & 1, abort_flag)) {
+      if ((threadIdx.x & 31) == leader) record_failure(abort_flag, L.status, kStatusTimeout);
       break;
     }
-    ptx::mbar_arrive_expect_tx(bar(C::B_VF + s), C::KV_BYTES);
+    if (ptx::elect_one(leader)) {
+      ptx::mbar_arrive_expect_tx(bar(C::B_VF + s), C::KV_BYTES);
 #pragma unroll
-    for (int kb = 0; kb < C::KB; ++kb)
-      ptx::tma_load_3d(sbase + C::OFF_V + s * C::KV_BYTES + kb * C::KV_BLOCK, &L.tm_v, bar(C::B_VF + s), kb * 64,
-                       g, kv.start, pol_kv);
+      for (int kb = 0; kb < C::KB; ++kb)
+        ptx::tma_load_3d(sbase + C::OFF_V + s * C::KV_BYTES + kb * C::KV_BLOCK, &L.tm_v, bar(C::B_VF + s), kb * 64,
+                         g, kv_start, pol_kv);
+    }
+    __syncwarp();
     v_issued = j + 1;
   }
   {
@@ -148,84 +184,149 @@ __device__ __forceinline__ void producer(const ProbeLaunch& L, const WorkItem& i
   }
 }
 
+// The whole warp walks the tiles on warp-uniform values; one elected lane
+// issues every MMA and commit. tcgen05.commit tracks the MMAs of the thread
+// that issues it, so the lane must not change: elect.sync picks the same lane
+// of a converged warp, and a change is treated as a failure.
 template <int TILE, int D, int NS>
-__device__ __forceinline__ void mma_issuer(const ProbeLaunch& L, const WorkItem& it, uint32_t sbase, uint32_t tmem,
-                                           volatile int* abort_flag) {
+__device__ __forceinline__ void mma_issuer(const ProbeLaunch& L, const WorkItem& it, uint32_t sbase_in,
+                                           uint32_t tmem_in, volatile int* abort_flag) {
   using C = Cfg<TILE, D, NS>;
+  const uint32_t sbase = __shfl_sync(0xffffffffu, sbase_in, 0);
+  const uint32_t tmem = __shfl_sync(0xffffffffu, tmem_in, 0);
+  const int n = __shfl_sync(0xffffffffu, it.kv_count, 0);
+  const bool two = heads_left(L, __shfl_sync(0xffffffffu, it.head, 0)) > C::HP;
   auto bar = [&](int i) { return sbase + C::OFF_BAR + 8u * i; };
   constexpr uint32_t kIdescS = ptx::idesc_bf16_f32(kRows, TILE, false, false);
   constexpr uint32_t kIdescO = ptx::idesc_bf16_f32(kRows, D, false, true);
-  const int n = it.kv_count;
-  bool ok = ptx::mbar_wait(bar(C::B_Q), 0, abort_flag, kWaitTimeoutNs);
-
-  auto issue_s = [&](int j) -> bool {
-    const int s = j % NS;
-    const int b = j & 1;
-    if (!ptx::mbar_wait(bar(C::B_KF + s), (j / NS) & 1, abort_flag, kWaitTimeoutNs)) return false;
-    ptx::tc_fence_after();
-    const uint32_t kbase = sbase + C::OFF_K + s * C::KV_BYTES;
+  uint32_t leader = 0;
+  int first_leader = -1;
+  bool same_leader = true;
+  auto elect = [&]() -> bool {
+    const bool me = ptx::elect_one(leader);
+    if (first_leader < 0) first_leader = static_cast<int>(leader);
+    same_leader = same_leader && static_cast<int>(leader) == first_leader;
+    return me && same_leader;
+  };
+  // S_slot = Q_slot K_j^T
+  auto mma_s = [&](int slot, int j) {
+    const uint32_t kbase = sbase + C::OFF_K + (j % NS) * C::KV_BYTES;
+    const uint32_t qbase = sbase + C::OFF_Q + slot * C::Q_BYTES;
 #pragma unroll
     for (int kk = 0; kk < D / 16; ++kk) {
-      const uint64_t a = ptx::sdesc_sw128(sbase + C::OFF_Q + (kk / 4) * C::Q_BLOCK + (kk % 4) * 32, 16, 1024);
+      const uint64_t a = ptx::sdesc_sw128(qbase + (kk / 4) * C::Q_BLOCK + (kk % 4) * 32, 16, 1024);
       const uint64_t bd = ptx::sdesc_sw128(kbase + (kk / 4) * C::KV_BLOCK + (kk % 4) * 32, 16, 1024);
-      ptx::mma_ss(tmem + C::COL_S0 + b * TILE, a, bd, kIdescS, kk > 0 ? 1u : 0u);
+      ptx::mma_ss(tmem + slot * C::SLOT_COLS + C::COL_S, a, bd, kIdescS, kk > 0 ? 1u : 0u);
     }
-    ptx::mma_commit(bar(C::B_SF + b));
-    ptx::mma_commit(bar(C::B_KE + s));
-    return true;
+  };
+  // O_slot += P_slot V_j, P from the first TILE/2 columns of the slot's S.
+  auto mma_pv = [&](int slot, int j) {
+    const uint32_t vbase = sbase + C::OFF_V + (j % NS) * C::KV_BYTES;
+#pragma unroll
+    for (int kk = 0; kk < TILE / 16; ++kk) {
+      const uint64_t bd = ptx::sdesc_sw128(vbase + kk * 16 * 128, C::KV_BLOCK, 1024);
+      ptx::mma_ts(tmem + slot * C::SLOT_COLS + C::COL_O, tmem + slot * C::SLOT_COLS + C::COL_S + kk * 8, bd, kIdescO,
+                  (j > 0 || kk > 0) ? 1u : 0u);
+    }
   };
 
+  bool issued = false;
+  bool ok = warp_wait(bar(C::B_Q), 0, abort_flag) && warp_wait(bar(C::B_KF), 0, abort_flag);
   if (ok) {
     ptx::tc_fence_after();
-    ok = issue_s(0);
+    if (elect()) {
+      mma_s(0, 0);
+      ptx::mma_commit(bar(C::B_SF));
+      if (two) {
+        mma_s(1, 0);
+        ptx::mma_commit(bar(C::B_SF + 1));
+      }
+      ptx::mma_commit(bar(C::B_KE));
+    }
+    __syncwarp();
+    issued = true;
+    ok = same_leader;
   }
   for (int j = 0; ok && j < n; ++j) {
-    if (j + 1 < n && !(ok = issue_s(j + 1))) break;
     const int s = j % NS;
-    const int b = j & 1;
-    if (!ptx::mbar_wait(bar(C::B_PF + b), (j >> 1) & 1, abort_flag, kWaitTimeoutNs) ||
-        !ptx::mbar_wait(bar(C::B_VF + s), (j / NS) & 1, abort_flag, kWaitTimeoutNs)) {
+    const int s1 = (j + 1) % NS;
+    const bool more = j + 1 < n;
+    // The K/V tiles landed long ago in steady state: test them before P0 so
+    // that P0's arrival starts P0.V and the next S0 at once.
+    if ((more && !warp_wait(bar(C::B_KF + s1), ((j + 1) / NS) & 1, abort_flag)) ||
+        !warp_wait(bar(C::B_VF + s), (j / NS) & 1, abort_flag) || !warp_wait(bar(C::B_PF), j & 1, abort_flag)) {
       ok = false;
       break;
     }
     ptx::tc_fence_after();
-    const uint32_t vbase = sbase + C::OFF_V + s * C::KV_BYTES;
-#pragma unroll
-    for (int kk = 0; kk < TILE / 16; ++kk) {
-      const uint64_t bd = ptx::sdesc_sw128(vbase + kk * 16 * 128, C::KV_BLOCK, 1024);
-      ptx::mma_ts(tmem + C::COL_O, tmem + C::COL_P0 + b * (TILE / 2) + kk * 8, bd, kIdescO,
-                  (j > 0 || kk > 0) ? 1u : 0u);
+    // slot 0: P.V of tile j, then S of tile j + 1
+    if (elect()) {
+      mma_pv(0, j);
+      if (!more) ptx::mma_commit(bar(C::B_OF));
+      if (more) {
+        mma_s(0, j + 1);
+        ptx::mma_commit(bar(C::B_SF));
+      }
     }
-    ptx::mma_commit(bar(C::B_PV + b));
-    ptx::mma_commit(bar(C::B_VE + s));
+    __syncwarp();
+    // slot 1: P.V of tile j, then S of tile j + 1
+    if (two) {
+      if (!warp_wait(bar(C::B_PF + 1), j & 1, abort_flag)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+    }
+    if (elect()) {
+      if (two) {
+        mma_pv(1, j);
+        if (!more) ptx::mma_commit(bar(C::B_OF + 1));
+      }
+      ptx::mma_commit(bar(C::B_VE + s));
+      if (more) {
+        if (two) {
+          mma_s(1, j + 1);
+          ptx::mma_commit(bar(C::B_SF + 1));
+        }
+        ptx::mma_commit(bar(C::B_KE + s1));
+      }
+    }
+    __syncwarp();
+    ok = same_leader;
   }
-  if (ok) {
-    ptx::mma_commit(bar(C::B_OF));
-  } else {
-    record_failure(abort_flag, L.status, kStatusTimeout);
-    // Wait for every MMA this thread issued before TMEM is released.
-    const volatile int never = 0;
-    ptx::mma_commit(bar(C::B_DRAIN));
-    ptx::mbar_wait(bar(C::B_DRAIN), 0, &never, kWaitTimeoutNs);
+  const int lane = threadIdx.x & 31;
+  if (!ok) {
+    if (lane == 0) record_failure(abort_flag, L.status, kStatusTimeout);
+    // Wait for every MMA the issuing lane started before TMEM is released.
+    if (issued && lane == first_leader) {
+      const volatile int never = 0;
+      ptx::mma_commit(bar(C::B_DRAIN));
+      ptx::mbar_wait(bar(C::B_DRAIN), 0, &never, kWaitTimeoutNs);
+    }
   }
+  __syncwarp();
 }
 
 template <int TILE, int D, int NS>
-__device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const WorkItem& it, uint32_t sbase,
-                                                 uint32_t tmem, volatile int* abort_flag) {
+__device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const WorkItem& it, int slot, uint32_t sbase,
+                                                 uint32_t tmem_base, volatile int* abort_flag) {
   using C = Cfg<TILE, D, NS>;
   auto bar = [&](int i) { return sbase + C::OFF_BAR + 8u * i; };
-  const int warp = threadIdx.x >> 5;
-  const int row = threadIdx.x;                 // TMEM lane
+  const int left = heads_left(L, it.head);
+  if (slot * C::HP >= left) return;            // the item has one slot only
+  const int warp = (threadIdx.x >> 5) & 3;
+  const int row = threadIdx.x & 127;           // TMEM lane
   const int hp = row / TILE;
   const int row_local = row % TILE;
-  const int gq = L.hq / L.hkv;
-  const bool head_ok = (hp == 0) || ((it.head + 1) < L.hq && (it.head + 1) / gq == it.head / gq);
-  const int head = it.head + hp;
+  const bool head_ok = slot * C::HP + hp < left;
+  const int head = it.head + slot * C::HP + hp;
   const bool row_ok = head_ok && row_local < it.q_len;
   const int qpos = it.q_start + row_local;
   const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+  const uint32_t tmem = tmem_base + lane_base + slot * C::SLOT_COLS;
   const bool spill_rows = it.text_row0 >= 0 && row_ok;
+  const uint32_t bar_sf = bar(C::B_SF + slot);
+  const uint32_t bar_pf = bar(C::B_PF + slot);
 
   float* spill_row = nullptr;
   int vis_start = 0;
@@ -240,53 +341,61 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
   float m_used = -INFINITY;   // running max, log2 units
   float l_sum = 0.f;
   bool ok = true;
+  const uint64_t scale2 = ptx::f2(L.scale_log2, L.scale_log2);
 
   for (int j = 0; j < it.kv_count; ++j) {
-    const int b = j & 1;
     const KvTile kv = L.kv[it.kv_begin + j];
-    if (!warp_wait(bar(C::B_SF + b), (j >> 1) & 1, abort_flag)) { ok = false; break; }
+    if (!warp_wait(bar_sf, j & 1, abort_flag)) { ok = false; break; }
     ptx::tc_fence_after();
-    float s[TILE];
-#pragma unroll
-    for (int c = 0; c < TILE / 32; ++c) {
-      uint32_t r[32];
-      ptx::tmem_ld32(tmem + lane_base + C::COL_S0 + b * TILE + c * 32, r);
-#pragma unroll
-      for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(r[e]);
+    // Keys past the tile's end (ragged tile) or above the diagonal are masked.
+    int limit = TILE;
+    if (kv.diag || kv.len < TILE) {
+      limit = kv.len;
+      if (kv.diag) limit = min(limit, qpos - kv.start + 1);
     }
-    ptx::tmem_wait_ld();
+    const bool spill = spill_rows && kv.visual;
+    float* spill_dst = spill ? spill_row + (kv.start - vis_start) : nullptr;
 
-    // Text rows keep their natural-log logits onto visual keys for the evidence pass.
-    if (spill_rows && kv.visual) {
-      float* dst = spill_row + (kv.start - vis_start);
-      const int n4 = (kv.len + 3) >> 2;
+    // Pass 1: row max (and the text rows' logit spill), 64 columns at a time.
+    float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int c4 = 0; c4 < TILE / 4; ++c4) {
-        if (c4 < n4) {
-          float4 w = make_float4(s[4 * c4] * L.scale, s[4 * c4 + 1] * L.scale, s[4 * c4 + 2] * L.scale,
-                                 s[4 * c4 + 3] * L.scale);
-          __stcs(reinterpret_cast<float4*>(dst) + c4, w);
+    for (int h = 0; h < TILE / 64; ++h) {
+      float s[64];
+      {
+        uint32_t r0[32], r1[32];
+        ptx::tmem_ld32(tmem + C::COL_S + h * 64, r0);
+        ptx::tmem_ld32(tmem + C::COL_S + h * 64 + 32, r1);
+        ptx::tmem_wait_ld();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          s[e] = __uint_as_float(r0[e]);
+          s[32 + e] = __uint_as_float(r1[e]);
         }
       }
-    }
-
-    if (kv.diag || kv.len < TILE) {
-      int limit = kv.len;
-      if (kv.diag) limit = min(limit, qpos - kv.start + 1);
+      if (spill) {
+        const int n4 = (kv.len + 3) >> 2;
 #pragma unroll
-      for (int c = 0; c < TILE; ++c) s[c] = c < limit ? s[c] : -INFINITY;
-    }
-    float m4[4] = {s[0], s[1], s[2], s[3]};
+        for (int c4 = 0; c4 < 16; ++c4) {
+          if (h * 16 + c4 < n4) {
+            float4 w = make_float4(s[4 * c4] * L.scale, s[4 * c4 + 1] * L.scale, s[4 * c4 + 2] * L.scale,
+                                   s[4 * c4 + 3] * L.scale);
+            __stcs(reinterpret_cast<float4*>(spill_dst) + h * 16 + c4, w);
+          }
+        }
+      }
+      if (limit < TILE) {
 #pragma unroll
-    for (int c = 4; c < TILE - 4; c += 8) {
-      m4[0] = ptx::max3(m4[0], s[c], s[c + 1]);
-      m4[1] = ptx::max3(m4[1], s[c + 2], s[c + 3]);
-      m4[2] = ptx::max3(m4[2], s[c + 4], s[c + 5]);
-      m4[3] = ptx::max3(m4[3], s[c + 6], s[c + 7]);
+        for (int c = 0; c < 64; ++c) s[c] = h * 64 + c < limit ? s[c] : -INFINITY;
+      }
+#pragma unroll
+      for (int c = 0; c < 64; c += 8) {
+        m4[0] = ptx::max3(m4[0], s[c], s[c + 1]);
+        m4[1] = ptx::max3(m4[1], s[c + 2], s[c + 3]);
+        m4[2] = ptx::max3(m4[2], s[c + 4], s[c + 5]);
+        m4[3] = ptx::max3(m4[3], s[c + 6], s[c + 7]);
+      }
     }
-    m4[0] = ptx::max3(m4[0], s[TILE - 4], s[TILE - 3]);
-    m4[1] = ptx::max3(m4[1], s[TILE - 2], s[TILE - 1]);
-    const float mx = ptx::max3(m4[0], m4[1], fmaxf(m4[2], m4[3]));
+    const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
     const float m_tile = mx * L.scale_log2;
     const bool need = m_tile > m_used + kRescaleThreshold;
     float alpha = 1.f;
@@ -297,27 +406,54 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
     }
     const float m_safe = (m_used == -INFINITY) ? 0.f : m_used;
 
-    // P buffer b was last read by PV_{j-2}.
-    if (j >= 2 && !warp_wait(bar(C::B_PV + b), ((j - 2) >> 1) & 1, abort_flag)) {
-      ok = false;
-      break;
+    // Lazy rescale of the O accumulator (only rows whose max moved by > 2^8).
+    // S_j was issued after P_{j-1}.V, so that MMA has completed.
+    if (j > 0 && __any_sync(0xffffffffu, need)) {
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t r[32];
+        ptx::tmem_ld32(tmem + C::COL_O + c * 32, r);
+        ptx::tmem_wait_ld();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+        ptx::tmem_st32(tmem + C::COL_O + c * 32, r);
+      }
     }
-    const uint64_t scale2 = ptx::f2(L.scale_log2, L.scale_log2);
+
+    // Pass 2: P = 2^(s * scale * log2 e - m) in packed pairs, written as bf16
+    // over the first half of S (columns of a 64-wide chunk are read before
+    // the chunk's P is stored, and P of chunk h lands below chunk h + 1).
     const uint64_t negm2 = ptx::f2(-m_safe, -m_safe);
     uint64_t l2[4] = {0, 0, 0, 0};
 #pragma unroll
-    for (int c = 0; c < TILE / 64; ++c) {
+    for (int h = 0; h < TILE / 64; ++h) {
+      float s[64];
+      {
+        uint32_t r0[32], r1[32];
+        ptx::tmem_ld32(tmem + C::COL_S + h * 64, r0);
+        ptx::tmem_ld32(tmem + C::COL_S + h * 64 + 32, r1);
+        ptx::tmem_wait_ld();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          s[e] = __uint_as_float(r0[e]);
+          s[32 + e] = __uint_as_float(r1[e]);
+        }
+      }
+      if (limit < TILE) {
+#pragma unroll
+        for (int c = 0; c < 64; ++c) s[c] = h * 64 + c < limit ? s[c] : -INFINITY;
+      }
       uint32_t pk[32];
 #pragma unroll
       for (int e = 0; e < 32; ++e) {
         float x0, x1;
-        ptx::unf2(ptx::fma2(ptx::f2(s[c * 64 + 2 * e], s[c * 64 + 2 * e + 1]), scale2, negm2), x0, x1);
+        ptx::unf2(ptx::fma2(ptx::f2(s[2 * e], s[2 * e + 1]), scale2, negm2), x0, x1);
         const float p0 = ptx::ex2(x0);
         const float p1 = ptx::ex2(x1);
         l2[e & 3] = ptx::add2(l2[e & 3], ptx::f2(p0, p1));
         pk[e] = ptx::pack_bf16x2(p0, p1);
       }
-      ptx::tmem_st32(tmem + lane_base + C::COL_P0 + b * (TILE / 2) + c * 32, pk);
+      ptx::tmem_st32(tmem + C::COL_S + h * 32, pk);
     }
     {
       float a0, a1, b0, b1, c0, c1, d0, d1;
@@ -327,34 +463,16 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
       ptx::unf2(l2[3], d0, d1);
       l_sum += ((a0 + a1) + (b0 + b1)) + ((c0 + c1) + (d0 + d1));
     }
-
-    // Lazy rescale of the O accumulator (only rows whose max moved by > 2^8).
-    if (j > 0 && __any_sync(0xffffffffu, need)) {
-      if (!warp_wait(bar(C::B_PV + ((j - 1) & 1)), ((j - 1) >> 1) & 1, abort_flag)) {
-        ok = false;
-        break;
-      }
-      ptx::tc_fence_after();
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
-        uint32_t r[32];
-        ptx::tmem_ld32(tmem + lane_base + C::COL_O + c * 32, r);
-        ptx::tmem_wait_ld();
-#pragma unroll
-        for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-        ptx::tmem_st32(tmem + lane_base + C::COL_O + c * 32, r);
-      }
-    }
     ptx::tmem_wait_st();
     ptx::tc_fence_before();
-    ptx::mbar_arrive(bar(C::B_PF + b));
+    ptx::mbar_arrive(bar_pf);
   }
 
   if (!ok) {
     record_failure(abort_flag, L.status, kStatusTimeout);
     return;
   }
-  if (!warp_wait(bar(C::B_OF), 0, abort_flag)) {
+  if (!warp_wait(bar(C::B_OF + slot), 0, abort_flag)) {
     record_failure(abort_flag, L.status, kStatusTimeout);
     return;
   }
@@ -367,7 +485,7 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
 #pragma unroll
     for (int c = 0; c < D / 32; ++c) {
       uint32_t r[32];
-      ptx::tmem_ld32(tmem + lane_base + C::COL_O + c * 32, r);
+      ptx::tmem_ld32(tmem + C::COL_O + c * 32, r);
       ptx::tmem_wait_ld();
       if (row_ok) {
 #pragma unroll
@@ -383,18 +501,19 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
     }
     if (row_ok) L.lse[static_cast<int64_t>(head) * L.n_tok + qpos] = (m_used + __log2f(l_sum)) * kLn2;
   } else {
-    float4* dst = reinterpret_cast<float4*>(L.part_o + (static_cast<int64_t>(it.part) * kRows + row) * D);
+    const int64_t part = it.part + slot;
+    float4* dst = reinterpret_cast<float4*>(L.part_o + (part * kRows + row) * D);
 #pragma unroll
     for (int c = 0; c < D / 32; ++c) {
       uint32_t r[32];
-      ptx::tmem_ld32(tmem + lane_base + C::COL_O + c * 32, r);
+      ptx::tmem_ld32(tmem + C::COL_O + c * 32, r);
       ptx::tmem_wait_ld();
 #pragma unroll
       for (int q4 = 0; q4 < 8; ++q4)
         dst[c * 8 + q4] = make_float4(__uint_as_float(r[4 * q4]), __uint_as_float(r[4 * q4 + 1]),
                                       __uint_as_float(r[4 * q4 + 2]), __uint_as_float(r[4 * q4 + 3]));
     }
-    L.part_ml[static_cast<int64_t>(it.part) * kRows + row] = make_float2(m_used, l_sum);
+    L.part_ml[part * kRows + row] = make_float2(m_used, l_sum);
   }
 }
 
@@ -407,7 +526,6 @@ __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_co
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
   const int warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
   const WorkItem it = L.items[blockIdx.x];
 
   if (threadIdx.x == 0) {
@@ -427,12 +545,12 @@ __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_co
   ptx::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 4) {
-    if (lane == 0) producer<TILE, D, NS>(L, it, sbase, abort_flag);
-  } else if (warp == 5) {
-    if (lane == 0) mma_issuer<TILE, D, NS>(L, it, sbase, tmem, abort_flag);
+  if (warp == kWarpProducer) {
+    producer<TILE, D, NS>(L, it, sbase, abort_flag);
+  } else if (warp == kWarpMma) {
+    mma_issuer<TILE, D, NS>(L, it, sbase, tmem, abort_flag);
   } else {
-    softmax_epilogue<TILE, D, NS>(L, it, sbase, tmem, abort_flag);
+    softmax_epilogue<TILE, D, NS>(L, it, warp / 4, sbase, tmem, abort_flag);
   }
   ptx::tc_fence_before();
   __syncthreads();

@@ -61,6 +61,18 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const v
   }
 }
 
+// ---------------------------------------------------------------- warp
+// Elects one lane of a converged warp (elect.sync); every lane learns which
+// one through a ballot.
+__device__ __forceinline__ bool elect_one(uint32_t& leader) {
+  uint32_t pred;
+  asm volatile(
+      "{\n\t.reg .pred P;\n\telect.sync _|P, 0xffffffff;\n\tselp.b32 %0, 1, 0, P;\n\t}"
+      : "=r"(pred));
+  leader = static_cast<uint32_t>(__ffs(__ballot_sync(0xffffffffu, pred != 0)) - 1);
+  return pred != 0;
+}
+
 // ---------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
