@@ -8,10 +8,12 @@
 // slots use every K/V tile the CTA loads, and each slot's softmax runs while
 // the tensor core works on the other slot.
 //
-// Warp roles (320 threads):
+// Warp roles (352 threads):
 //   warps 0-3  softmax + epilogue of slot 0, one thread per query row (TMEM lane)
 //   warps 4-7  softmax + epilogue of slot 1
-//   warp 8     TMA producer: Q of both slots, then K_j / V_j into NS-deep rings
+//   warp 8     TMA: Q of both slots, then K_j into an NS-deep ring
+//   warp 10    TMA: V_j into an NS-deep ring (apart from K, so that K tiles
+//              run ahead of the V waits)
 //   warp 9     MMA issuer; the warp walks the tiles together and one elected
 //              lane issues, per kv tile j:
 //                O0 += P0_j V_j,  S0_{j+1} = Q0 K_{j+1}^T,
@@ -19,7 +21,9 @@
 // TMEM columns per slot: S (TILE) | O (D). P_j (bf16) is written over the
 // first half of its own S_j columns and read from there by the P.V MMA; the
 // slot's next S is issued after that P.V, and the tcgen05 MMAs of one thread
-// execute in issue order.
+// execute in issue order. An item with one slot (the last heads of a KV group
+// with an odd head count) uses the idle slot's S columns as a second S
+// buffer: S_{j+1} is computed while the softmax works on S_j.
 // Online softmax in fp32 (log2 domain) with lazy rescaling: the running max is
 // only moved when it grows by more than 2^8, so O in TMEM is rescaled rarely.
 // Text row tiles also spill their logits onto visual keys for the evidence
@@ -35,9 +39,10 @@ namespace evisel {
 namespace {
 
 static_assert(kSlots == 2, "the kernel runs two slots per work item");
-constexpr int kThreads = 320;
-constexpr int kWarpProducer = 8;
+constexpr int kThreads = 352;
+constexpr int kWarpProducer = 8;   // Q, then the K ring
 constexpr int kWarpMma = 9;
+constexpr int kWarpVLoader = 10;   // the V ring
 constexpr int kRows = 128;
 constexpr float kRescaleThreshold = 8.0f;   // log2 units
 constexpr float kLn2 = 0.69314718055994531f;
@@ -98,7 +103,9 @@ __device__ __forceinline__ int heads_left(const ProbeLaunch& L, int head) {
   return gq - head % gq;
 }
 
-template <int TILE, int D, int NS>
+// One TMA warp per ring, so that K tiles run ahead of the V waits: the K warp
+// also loads Q, the V warp only its ring.
+template <int TILE, int D, int NS, bool IS_V>
 __device__ __forceinline__ void producer(const ProbeLaunch& L, const WorkItem& it, uint32_t sbase_in,
                                          volatile int* abort_flag) {
   using C = Cfg<TILE, D, NS>;
@@ -114,7 +121,7 @@ __device__ __forceinline__ void producer(const ProbeLaunch& L, const WorkItem& i
   const uint64_t pol_q = ptx::l2_policy_evict_first();
   const uint64_t pol_kv = ptx::l2_policy_evict_last();
   uint32_t leader = 0;
-  if (ptx::elect_one(leader)) {
+  if (!IS_V && ptx::elect_one(leader)) {
     ptx::tma_prefetch_desc(&L.tm_q);
     ptx::tma_prefetch_desc(&L.tm_k);
     ptx::tma_prefetch_desc(&L.tm_v);
@@ -133,53 +140,38 @@ __device__ __forceinline__ void producer(const ProbeLaunch& L, const WorkItem& i
   }
   __syncwarp();
 
-  int k_issued = 0, v_issued = 0;
+  const CUtensorMap* map = IS_V ? &L.tm_v : &L.tm_k;
+  const int off = IS_V ? C::OFF_V : C::OFF_K;
+  const int b_full = IS_V ? C::B_VF : C::B_KF;
+  const int b_empty = IS_V ? C::B_VE : C::B_KE;
+  int issued = 0;
   for (int j = 0; j < n; ++j) {
     const int s = j % NS;
     const int u = j / NS;
     const int kv_start = __shfl_sync(0xffffffffu, L.kv[kv_begin + j].start, 0);
-    if (u > 0 && !warp_wait(bar(C::B_KE + s), (u - 1) & 1, abort_flag)) {
+    if (u > 0 && !warp_wait(bar(b_empty + s), (u - 1) & 1, abort_flag)) {
       if ((threadIdx.x & 31) == leader) record_failure(abort_flag, L.status, kStatusTimeout);
       break;
     }
     if (ptx::elect_one(leader)) {
-      ptx::mbar_arrive_expect_tx(bar(C::B_KF + s), C::KV_BYTES);
+      ptx::mbar_arrive_expect_tx(bar(b_full + s), C::KV_BYTES);
 #pragma unroll
       for (int kb = 0; kb < C::KB; ++kb)
-        ptx::tma_load_3d(sbase + C::OFF_K + s * C::KV_BYTES + kb * C::KV_BLOCK, &L.tm_k, bar(C::B_KF + s), kb * 64,
-                         g, kv_start, pol_kv);
+        ptx::tma_load_3d(sbase + off + s * C::KV_BYTES + kb * C::KV_BLOCK, map, bar(b_full + s), kb * 64, g, kv_start,
+                         pol_kv);
     }
     __syncwarp();
-    k_issued = j + 1;
-    if (u > 0 && !warp_wait(bar(C::B_VE + s), (u - 1) & 1, abort_flag)) {
-      if ((threadIdx.x & 31) == leader) record_failure(abort_flag, L.status, kStatusTimeout);
-      break;
-    }
-    if (ptx::elect_one(leader)) {
-      ptx::mbar_arrive_expect_tx(bar(C::B_VF + s), C::KV_BYTES);
-#pragma unroll
-      for (int kb = 0; kb < C::KB; ++kb)
-        ptx::tma_load_3d(sbase + C::OFF_V + s * C::KV_BYTES + kb * C::KV_BLOCK, &L.tm_v, bar(C::B_VF + s), kb * 64,
-                         g, kv_start, pol_kv);
-    }
-    __syncwarp();
-    v_issued = j + 1;
+    issued = j + 1;
   }
   {
     // Drain: every load issued here completes on its own; wait for the last
     // phase issued into each stage (and for Q) so that no copy is in flight
     // when the CTA exits, whether or not another warp gave up.
     const volatile int never = 0;
-    ptx::mbar_wait(bar(C::B_Q), 0, &never, kWaitTimeoutNs);
-    for (int s = 0; s < NS; ++s) {
-      if (s < k_issued) {
-        const int last = ((k_issued - 1 - s) / NS) * NS + s;
-        ptx::mbar_wait(bar(C::B_KF + s), (last / NS) & 1, &never, kWaitTimeoutNs);
-      }
-      if (s < v_issued) {
-        const int last = ((v_issued - 1 - s) / NS) * NS + s;
-        ptx::mbar_wait(bar(C::B_VF + s), (last / NS) & 1, &never, kWaitTimeoutNs);
-      }
+    if (!IS_V) ptx::mbar_wait(bar(C::B_Q), 0, &never, kWaitTimeoutNs);
+    for (int s = 0; s < NS && s < issued; ++s) {
+      const int last = ((issued - 1 - s) / NS) * NS + s;
+      ptx::mbar_wait(bar(b_full + s), (last / NS) & 1, &never, kWaitTimeoutNs);
     }
   }
 }
@@ -208,91 +200,138 @@ __device__ __forceinline__ void mma_issuer(const ProbeLaunch& L, const WorkItem&
     same_leader = same_leader && static_cast<int>(leader) == first_leader;
     return me && same_leader;
   };
-  // S_slot = Q_slot K_j^T
-  auto mma_s = [&](int slot, int j) {
+  // S[buf] = Q_slot K_j^T (buf: whose S columns receive it)
+  auto mma_s = [&](int slot, int j, int buf) {
     const uint32_t kbase = sbase + C::OFF_K + (j % NS) * C::KV_BYTES;
     const uint32_t qbase = sbase + C::OFF_Q + slot * C::Q_BYTES;
 #pragma unroll
     for (int kk = 0; kk < D / 16; ++kk) {
       const uint64_t a = ptx::sdesc_sw128(qbase + (kk / 4) * C::Q_BLOCK + (kk % 4) * 32, 16, 1024);
       const uint64_t bd = ptx::sdesc_sw128(kbase + (kk / 4) * C::KV_BLOCK + (kk % 4) * 32, 16, 1024);
-      ptx::mma_ss(tmem + slot * C::SLOT_COLS + C::COL_S, a, bd, kIdescS, kk > 0 ? 1u : 0u);
+      ptx::mma_ss(tmem + buf * C::SLOT_COLS + C::COL_S, a, bd, kIdescS, kk > 0 ? 1u : 0u);
     }
   };
-  // O_slot += P_slot V_j, P from the first TILE/2 columns of the slot's S.
-  auto mma_pv = [&](int slot, int j) {
+  // O_slot += P V_j, P from the first TILE/2 columns of S[buf].
+  auto mma_pv = [&](int slot, int j, int buf) {
     const uint32_t vbase = sbase + C::OFF_V + (j % NS) * C::KV_BYTES;
 #pragma unroll
     for (int kk = 0; kk < TILE / 16; ++kk) {
       const uint64_t bd = ptx::sdesc_sw128(vbase + kk * 16 * 128, C::KV_BLOCK, 1024);
-      ptx::mma_ts(tmem + slot * C::SLOT_COLS + C::COL_O, tmem + slot * C::SLOT_COLS + C::COL_S + kk * 8, bd, kIdescO,
+      ptx::mma_ts(tmem + slot * C::SLOT_COLS + C::COL_O, tmem + buf * C::SLOT_COLS + C::COL_S + kk * 8, bd, kIdescO,
                   (j > 0 || kk > 0) ? 1u : 0u);
     }
   };
 
   bool issued = false;
   bool ok = warp_wait(bar(C::B_Q), 0, abort_flag) && warp_wait(bar(C::B_KF), 0, abort_flag);
-  if (ok) {
-    ptx::tc_fence_after();
-    if (elect()) {
-      mma_s(0, 0);
-      ptx::mma_commit(bar(C::B_SF));
-      if (two) {
-        mma_s(1, 0);
-        ptx::mma_commit(bar(C::B_SF + 1));
-      }
-      ptx::mma_commit(bar(C::B_KE));
-    }
-    __syncwarp();
-    issued = true;
-    ok = same_leader;
-  }
-  for (int j = 0; ok && j < n; ++j) {
-    const int s = j % NS;
-    const int s1 = (j + 1) % NS;
-    const bool more = j + 1 < n;
-    // The K/V tiles landed long ago in steady state: test them before P0 so
-    // that P0's arrival starts P0.V and the next S0 at once.
-    if ((more && !warp_wait(bar(C::B_KF + s1), ((j + 1) / NS) & 1, abort_flag)) ||
-        !warp_wait(bar(C::B_VF + s), (j / NS) & 1, abort_flag) || !warp_wait(bar(C::B_PF), j & 1, abort_flag)) {
-      ok = false;
-      break;
-    }
-    ptx::tc_fence_after();
-    // slot 0: P.V of tile j, then S of tile j + 1
-    if (elect()) {
-      mma_pv(0, j);
-      if (!more) ptx::mma_commit(bar(C::B_OF));
-      if (more) {
-        mma_s(0, j + 1);
+  if (!two) {
+    // One slot: the second slot's S columns double-buffer S, so S_{j+1} is
+    // ready while the softmax works on S_j. Tile j uses buffer b = j & 1
+    // (barriers SF[b] / PF[b], phase j >> 1); S_{j+2} reuses b after P_j.V.
+    if (ok) {
+      ptx::tc_fence_after();
+      if (elect()) {
+        mma_s(0, 0, 0);
         ptx::mma_commit(bar(C::B_SF));
+        ptx::mma_commit(bar(C::B_KE));
+      }
+      __syncwarp();
+      issued = true;
+      ok = same_leader;
+    }
+    if (ok && n > 1) {
+      if (!warp_wait(bar(C::B_KF + 1 % NS), (1 / NS) & 1, abort_flag)) {
+        ok = false;
+      } else {
+        if (elect()) {
+          mma_s(0, 1, 1);
+          ptx::mma_commit(bar(C::B_SF + 1));
+          ptx::mma_commit(bar(C::B_KE + 1 % NS));
+        }
+        __syncwarp();
+        ok = same_leader;
       }
     }
-    __syncwarp();
-    // slot 1: P.V of tile j, then S of tile j + 1
-    if (two) {
+    for (int j = 0; ok && j < n; ++j) {
+      const int b = j & 1;
+      const int s = j % NS;
+      const int s2 = (j + 2) % NS;
+      const bool more = j + 2 < n;
+      if ((more && !warp_wait(bar(C::B_KF + s2), ((j + 2) / NS) & 1, abort_flag)) ||
+          !warp_wait(bar(C::B_VF + s), (j / NS) & 1, abort_flag) ||
+          !warp_wait(bar(C::B_PF + b), (j >> 1) & 1, abort_flag)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      if (elect()) {
+        mma_pv(0, j, b);
+        if (j + 1 == n) ptx::mma_commit(bar(C::B_OF));
+        ptx::mma_commit(bar(C::B_VE + s));
+        if (more) {
+          mma_s(0, j + 2, b);
+          ptx::mma_commit(bar(C::B_SF + b));
+          ptx::mma_commit(bar(C::B_KE + s2));
+        }
+      }
+      __syncwarp();
+      ok = same_leader;
+    }
+  } else {
+    if (ok) {
+      ptx::tc_fence_after();
+      if (elect()) {
+        mma_s(0, 0, 0);
+        ptx::mma_commit(bar(C::B_SF));
+        mma_s(1, 0, 1);
+        ptx::mma_commit(bar(C::B_SF + 1));
+        ptx::mma_commit(bar(C::B_KE));
+      }
+      __syncwarp();
+      issued = true;
+      ok = same_leader;
+    }
+    for (int j = 0; ok && j < n; ++j) {
+      const int s = j % NS;
+      const int s1 = (j + 1) % NS;
+      const bool more = j + 1 < n;
+      // The K/V tiles landed long ago in steady state: test them before P0 so
+      // that P0's arrival starts P0.V and the next S0 at once.
+      if ((more && !warp_wait(bar(C::B_KF + s1), ((j + 1) / NS) & 1, abort_flag)) ||
+          !warp_wait(bar(C::B_VF + s), (j / NS) & 1, abort_flag) || !warp_wait(bar(C::B_PF), j & 1, abort_flag)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      // slot 0: P.V of tile j, then S of tile j + 1
+      if (elect()) {
+        mma_pv(0, j, 0);
+        if (!more) ptx::mma_commit(bar(C::B_OF));
+        if (more) {
+          mma_s(0, j + 1, 0);
+          ptx::mma_commit(bar(C::B_SF));
+        }
+      }
+      __syncwarp();
+      // slot 1: P.V of tile j, then S of tile j + 1
       if (!warp_wait(bar(C::B_PF + 1), j & 1, abort_flag)) {
         ok = false;
         break;
       }
       ptx::tc_fence_after();
-    }
-    if (elect()) {
-      if (two) {
-        mma_pv(1, j);
+      if (elect()) {
+        mma_pv(1, j, 1);
         if (!more) ptx::mma_commit(bar(C::B_OF + 1));
-      }
-      ptx::mma_commit(bar(C::B_VE + s));
-      if (more) {
-        if (two) {
-          mma_s(1, j + 1);
+        ptx::mma_commit(bar(C::B_VE + s));
+        if (more) {
+          mma_s(1, j + 1, 1);
           ptx::mma_commit(bar(C::B_SF + 1));
+          ptx::mma_commit(bar(C::B_KE + s1));
         }
-        ptx::mma_commit(bar(C::B_KE + s1));
       }
+      __syncwarp();
+      ok = same_leader;
     }
-    __syncwarp();
-    ok = same_leader;
   }
   const int lane = threadIdx.x & 31;
   if (!ok) {
@@ -325,8 +364,8 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
   const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
   const uint32_t tmem = tmem_base + lane_base + slot * C::SLOT_COLS;
   const bool spill_rows = it.text_row0 >= 0 && row_ok;
-  const uint32_t bar_sf = bar(C::B_SF + slot);
-  const uint32_t bar_pf = bar(C::B_PF + slot);
+  // With one slot, S alternates between both slots' S columns (see the MMA issuer).
+  const bool two = left > C::HP;
 
   float* spill_row = nullptr;
   int vis_start = 0;
@@ -345,7 +384,11 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
 
   for (int j = 0; j < it.kv_count; ++j) {
     const KvTile kv = L.kv[it.kv_begin + j];
-    if (!warp_wait(bar_sf, j & 1, abort_flag)) { ok = false; break; }
+    const int b = two ? slot : (j & 1);
+    const uint32_t par = two ? (j & 1) : ((j >> 1) & 1);
+    const uint32_t tS = tmem_base + lane_base + b * C::SLOT_COLS + C::COL_S;
+    const uint32_t bar_pf = bar(C::B_PF + b);
+    if (!warp_wait(bar(C::B_SF + b), par, abort_flag)) { ok = false; break; }
     ptx::tc_fence_after();
     // Keys past the tile's end (ragged tile) or above the diagonal are masked.
     int limit = TILE;
@@ -363,8 +406,8 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
       float s[64];
       {
         uint32_t r0[32], r1[32];
-        ptx::tmem_ld32(tmem + C::COL_S + h * 64, r0);
-        ptx::tmem_ld32(tmem + C::COL_S + h * 64 + 32, r1);
+        ptx::tmem_ld32(tS + h * 64, r0);
+        ptx::tmem_ld32(tS + h * 64 + 32, r1);
         ptx::tmem_wait_ld();
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
@@ -407,8 +450,14 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
     const float m_safe = (m_used == -INFINITY) ? 0.f : m_used;
 
     // Lazy rescale of the O accumulator (only rows whose max moved by > 2^8).
-    // S_j was issued after P_{j-1}.V, so that MMA has completed.
+    // With two slots S_j was issued after P_{j-1}.V, so that MMA has
+    // completed; with one slot it is waited for (its V-empty barrier).
     if (j > 0 && __any_sync(0xffffffffu, need)) {
+      if (!two && !warp_wait(bar(C::B_VE + (j - 1) % NS), ((j - 1) / NS) & 1, abort_flag)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
         uint32_t r[32];
@@ -430,8 +479,8 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
       float s[64];
       {
         uint32_t r0[32], r1[32];
-        ptx::tmem_ld32(tmem + C::COL_S + h * 64, r0);
-        ptx::tmem_ld32(tmem + C::COL_S + h * 64 + 32, r1);
+        ptx::tmem_ld32(tS + h * 64, r0);
+        ptx::tmem_ld32(tS + h * 64 + 32, r1);
         ptx::tmem_wait_ld();
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
@@ -453,7 +502,7 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
         l2[e & 3] = ptx::add2(l2[e & 3], ptx::f2(p0, p1));
         pk[e] = ptx::pack_bf16x2(p0, p1);
       }
-      ptx::tmem_st32(tmem + C::COL_S + h * 32, pk);
+      ptx::tmem_st32(tS + h * 32, pk);
     }
     {
       float a0, a1, b0, b1, c0, c1, d0, d1;
@@ -546,7 +595,9 @@ __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_co
   const uint32_t tmem = *tmem_slot;
 
   if (warp == kWarpProducer) {
-    producer<TILE, D, NS>(L, it, sbase, abort_flag);
+    producer<TILE, D, NS, false>(L, it, sbase, abort_flag);
+  } else if (warp == kWarpVLoader) {
+    producer<TILE, D, NS, true>(L, it, sbase, abort_flag);
   } else if (warp == kWarpMma) {
     mma_issuer<TILE, D, NS>(L, it, sbase, tmem, abort_flag);
   } else {
