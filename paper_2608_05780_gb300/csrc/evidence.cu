@@ -3,10 +3,13 @@
 // evidence_reduce: re-forms the text-row probabilities P_im = exp(s_im - LSE_i)
 // from the spilled logits and the saved LSE and sums them over the text rows
 // (token map), then over each frame's N_v tokens (frame map). HBM-bound: one
-// streaming read of the spill. One block handles 128 visual columns of one
-// video for one head; its 8 warps split the text rows, each lane owns 4
-// consecutive columns (16-byte loads); partial sums meet in shared memory and
-// frames are closed with a segmented warp-shuffle sum (N_v / 4 lanes).
+// streaming read of the spill, laid out [hq, text rows / 32, n_vis, 32] (the
+// attention kernel writes one key of a warp's 32 rows as 128 contiguous
+// bytes). One block handles 128 visual keys of one video for one head: per
+// 32-row block those keys are 16 KB in a row; each of the 4 warps reads its
+// 32 keys' 4 KB with 16-byte loads (lane l: 4 rows of keys 4i + l / 8), sums
+// over all row blocks in registers, closes each key over its 8 lanes, and the
+// block forms the frames (N_v divides 128) from the 128 token sums.
 //
 // evidence_finalize: head map (sum of a video's frames per head) and the
 // query-frame cue A_qf (sum over heads / (Hq * n_text)), both recomputed from
@@ -19,77 +22,73 @@
 namespace evisel {
 namespace {
 
-constexpr int kWarps = 8;
-
-__device__ __forceinline__ float4 ld_stream(const float* p) {
-  return __ldcs(reinterpret_cast<const float4*>(p));
-}
+constexpr int kChunk = 128;                        // visual keys per block
+constexpr int kWarps = kChunk / 32;                // one warp per 32 keys
 
 __global__ void __launch_bounds__(kWarps * 32) evidence_reduce_kernel(const __grid_constant__ EvidenceLaunch L) {
-  __shared__ float4 part[kWarps][32];
+  __shared__ float tok_s[kChunk];
   const int h = blockIdx.y;
   const EvChunk ck = L.chunks[blockIdx.x];
   const VideoInfo vi = L.videos[ck.video];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int col = ck.col0 + lane * 4;            // visual column within the video
-  const bool col_ok = col < vi.n_vis;            // n_vis is a multiple of 4
+  const int n_rb = vi.text_pitch >> 5;
+  const float* lse = L.lse + static_cast<int64_t>(h) * L.n_tok + vi.vis_start + vi.n_vis;
+  const int key0 = ck.col0 + warp * 32;             // this warp's first key (within the video)
+  const int sub = lane & 7;                         // rows 4 sub .. 4 sub + 3 of each row block
+  // float4 i of the warp's 4 KB in a row block: keys key0 + 4 i + lane / 8.
+  const float4* base = reinterpret_cast<const float4*>(L.spill + vi.spill_off +
+                                                       static_cast<int64_t>(h) * vi.n_vis * vi.text_pitch +
+                                                       static_cast<int64_t>(key0) * 32) + lane;
 
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (col_ok) {
-    const float* base = L.spill + vi.spill_off + static_cast<int64_t>(h) * vi.n_text * vi.vis_pitch + col;
-    const float* lse = L.lse + static_cast<int64_t>(h) * L.n_tok + vi.vis_start + vi.n_vis;
-    int i = warp;
-    for (; i + 3 * kWarps < vi.n_text; i += 4 * kWarps) {
-      float4 s[4];
-      float m[4];
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  for (int rb = 0; rb < n_rb; ++rb) {
+    const int row = rb * 32 + 4 * sub;
+    float m[4];
+    bool in[4];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        s[u] = ld_stream(base + static_cast<int64_t>(i + u * kWarps) * vi.vis_pitch);
-        m[u] = __ldg(lse + i + u * kWarps);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        acc.x += __expf(s[u].x - m[u]);
-        acc.y += __expf(s[u].y - m[u]);
-        acc.z += __expf(s[u].z - m[u]);
-        acc.w += __expf(s[u].w - m[u]);
-      }
+    for (int u = 0; u < 4; ++u) {
+      in[u] = row + u < vi.n_text;   // rows past n_text are padding that was never written
+      m[u] = in[u] ? __ldg(lse + row + u) : 0.f;
     }
-    for (; i < vi.n_text; i += kWarps) {
-      const float4 s = ld_stream(base + static_cast<int64_t>(i) * vi.vis_pitch);
-      const float m = __ldg(lse + i);
-      acc.x += __expf(s.x - m);
-      acc.y += __expf(s.y - m);
-      acc.z += __expf(s.z - m);
-      acc.w += __expf(s.w - m);
+    const float4* src = base + static_cast<int64_t>(rb) * vi.n_vis * 8;
+    float4 sv[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      sv[i] = key0 + 4 * i + (lane >> 3) < vi.n_vis ? __ldcs(src + i * 32)
+                                                   : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float e0 = in[0] ? __expf(sv[i].x - m[0]) : 0.f;
+      const float e1 = in[1] ? __expf(sv[i].y - m[1]) : 0.f;
+      const float e2 = in[2] ? __expf(sv[i].z - m[2]) : 0.f;
+      const float e3 = in[3] ? __expf(sv[i].w - m[3]) : 0.f;
+      acc[i] += (e0 + e1) + (e2 + e3);
     }
   }
-  part[warp][lane] = acc;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    float t = acc[i];
+    t += __shfl_xor_sync(0xffffffffu, t, 4);
+    t += __shfl_xor_sync(0xffffffffu, t, 2);
+    t += __shfl_xor_sync(0xffffffffu, t, 1);
+    if (sub == 0) tok_s[warp * 32 + 4 * i + (lane >> 3)] = t;
+  }
   __syncthreads();
-  if (warp != 0) return;
-  float4 t = part[0][lane];
-#pragma unroll
-  for (int w = 1; w < kWarps; ++w) {
-    const float4 o = part[w][lane];
-    t.x += o.x; t.y += o.y; t.z += o.z; t.w += o.w;
-  }
+
+  const int nkeys = min(kChunk, vi.n_vis - ck.col0);   // a multiple of N_v
+  const int c = threadIdx.x;
   // Token map.
-  if (col_ok) {
-    float4* dst = reinterpret_cast<float4*>(L.tok + static_cast<int64_t>(h) * L.total_vis + vi.vis_off + col);
-    if (L.accumulate) {
-      const float4 o = *dst;
-      *dst = make_float4(o.x + t.x, o.y + t.y, o.z + t.z, o.w + t.w);
-    } else {
-      *dst = t;
-    }
+  if (c < nkeys) {
+    float* dst = L.tok + static_cast<int64_t>(h) * L.total_vis + vi.vis_off + ck.col0 + c;
+    *dst = L.accumulate ? *dst + tok_s[c] : tok_s[c];
   }
-  // Frame map: frames of N_v tokens are N_v / 4 consecutive lanes.
-  float f = t.x + t.y + t.z + t.w;
-  const int lanes = L.tokens_per_frame >> 2;
-  for (int off = 1; off < lanes; off <<= 1) f += __shfl_xor_sync(0xffffffffu, f, off);
-  if (col_ok && (lane & (lanes - 1)) == 0) {
-    float* dst = L.frame + static_cast<int64_t>(h) * L.total_frames + vi.frame_off + col / L.tokens_per_frame;
+  // Frame map: frame f of the chunk is keys [f N_v, (f + 1) N_v).
+  const int npf = L.tokens_per_frame;
+  if (c < nkeys / npf) {
+    float f = 0.f;
+    for (int i = 0; i < npf; ++i) f += tok_s[c * npf + i];
+    float* dst = L.frame + static_cast<int64_t>(h) * L.total_frames + vi.frame_off + ck.col0 / npf + c;
     *dst = L.accumulate ? *dst + f : f;
   }
 }

@@ -156,11 +156,11 @@ void build_plan(const evisel_probe_args* a, Plan& P) {
     v.vis_start = a->cu_seqlens_h[b];
     v.n_vis = a->n_vis_h[b];
     v.n_text = a->cu_seqlens_h[b + 1] - a->cu_seqlens_h[b] - v.n_vis;
-    v.vis_pitch = (v.n_vis + 3) & ~3;
+    v.text_pitch = (v.n_text + 31) & ~31;
     v.spill_off = spill;
     v.vis_off = vis_off;
     v.frame_off = frame_off;
-    spill += static_cast<int64_t>(hq) * v.n_text * v.vis_pitch;
+    spill += static_cast<int64_t>(hq) * v.n_vis * v.text_pitch;
     vis_off += v.n_vis;
     frame_off += v.n_vis / a->tokens_per_frame;
     P.videos.push_back(v);

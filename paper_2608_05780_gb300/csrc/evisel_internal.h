@@ -42,11 +42,11 @@ static_assert(sizeof(WorkItem) == 32, "WorkItem is 32 bytes");
 
 // Per-video layout used by the spill and the evidence pass.
 struct VideoInfo {
-  int64_t spill_off;  // float offset of this video's [hq, n_text, vis_pitch] logit block
+  int64_t spill_off;  // float offset of this video's logit block [hq, text_pitch / 32, n_vis, 32]
   int32_t vis_start;  // global index of its first visual token
   int32_t n_vis;
   int32_t n_text;
-  int32_t vis_pitch;  // n_vis rounded up to a multiple of 4 (row pitch of the spill)
+  int32_t text_pitch; // n_text rounded up to a multiple of 32 (rows of the spill, in blocks of 32)
   int32_t vis_off;    // column offset of its tokens in the token map
   int32_t frame_off;  // column offset of its frames in the frame map
 };

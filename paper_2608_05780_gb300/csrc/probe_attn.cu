@@ -372,9 +372,13 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
   if (it.text_row0 >= 0) {
     const VideoInfo vi = L.videos[it.video];
     vis_start = vi.vis_start;
-    if (row_ok)
-      spill_row = L.spill + vi.spill_off +
-                  (static_cast<int64_t>(head) * vi.n_text + it.text_row0 + row_local) * vi.vis_pitch;
+    // Spill [hq, text_pitch / 32, n_vis, 32]: a warp's 32 rows are one row
+    // block, and for one key they are 128 contiguous bytes.
+    if (row_ok) {
+      const int r = it.text_row0 + row_local;
+      spill_row = L.spill + vi.spill_off + static_cast<int64_t>(head) * vi.n_vis * vi.text_pitch +
+                  static_cast<int64_t>(r >> 5) * vi.n_vis * 32 + (r & 31);
+    }
   }
 
   float m_used = -INFINITY;   // running max, log2 units
@@ -397,7 +401,7 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
       if (kv.diag) limit = min(limit, qpos - kv.start + 1);
     }
     const bool spill = spill_rows && kv.visual;
-    float* spill_dst = spill ? spill_row + (kv.start - vis_start) : nullptr;
+    float* spill_dst = spill ? spill_row + static_cast<int64_t>(kv.start - vis_start) * 32 : nullptr;
 
     // Pass 1: row max (and the text rows' logit spill), 64 columns at a time.
     float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
@@ -416,15 +420,10 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
         }
       }
       if (spill) {
-        const int n4 = (kv.len + 3) >> 2;
+        float* dst = spill_dst + h * 64 * 32;
 #pragma unroll
-        for (int c4 = 0; c4 < 16; ++c4) {
-          if (h * 16 + c4 < n4) {
-            float4 w = make_float4(s[4 * c4] * L.scale, s[4 * c4 + 1] * L.scale, s[4 * c4 + 2] * L.scale,
-                                   s[4 * c4 + 3] * L.scale);
-            __stcs(reinterpret_cast<float4*>(spill_dst) + h * 16 + c4, w);
-          }
-        }
+        for (int c = 0; c < 64; ++c)
+          if (h * 64 + c < kv.len) __stcs(dst + c * 32, s[c] * L.scale);
       }
       if (limit < TILE) {
 #pragma unroll
