@@ -468,6 +468,7 @@ int evisel_probe_attention(const evisel_probe_args* args, void* stream_ptr, evis
     rc = encode_map(&L.tm_q, args->q, P.n_tok, args->hq, args->head_dim, args->tile);
     if (rc == EVISEL_OK) rc = encode_map(&L.tm_k, args->k, P.n_tok, args->hkv, args->head_dim, args->tile);
     if (rc == EVISEL_OK) rc = encode_map(&L.tm_v, args->v, P.n_tok, args->hkv, args->head_dim, args->tile);
+    if (rc == EVISEL_OK) rc = encode_map(&L.tm_o, args->o, P.n_tok, args->hq, args->head_dim, args->tile);
     if (rc != EVISEL_OK) return rc;
     L.items = ws->d_items;
     L.kv = ws->d_kv;

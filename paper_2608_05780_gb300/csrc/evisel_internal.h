@@ -73,6 +73,7 @@ struct EvChunk {
 
 struct ProbeLaunch {
   CUtensorMap tm_q, tm_k, tm_v;     // 3-D maps {d, heads, tokens}, box {64, 1, tile}, 128B swizzle
+  CUtensorMap tm_o;                 // O, laid out and boxed like Q (epilogue stores)
   const WorkItem* items;
   const KvTile* kv;
   const VideoInfo* videos;

@@ -248,6 +248,7 @@ extern "C" int evisel_probe_evidence_noalloc(const evisel_probe_args* args, floa
     rc = encode_tensor_map(&L.tm_q, args->q, n_tok, args->hq, args->head_dim, args->tile);
     if (rc == EVISEL_OK) rc = encode_tensor_map(&L.tm_k, args->k, n_tok, args->hkv, args->head_dim, args->tile);
     if (rc == EVISEL_OK) rc = encode_tensor_map(&L.tm_v, args->v, n_tok, args->hkv, args->head_dim, args->tile);
+    if (rc == EVISEL_OK) rc = encode_tensor_map(&L.tm_o, args->o, n_tok, args->hq, args->head_dim, args->tile);
     if (rc != EVISEL_OK) return rc;
     L.items = reinterpret_cast<const WorkItem*>(base + o_items);
     L.kv = reinterpret_cast<const KvTile*>(base + o_kv);

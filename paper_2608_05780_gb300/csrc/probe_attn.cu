@@ -527,7 +527,47 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
   ptx::tc_fence_after();
 
   const float inv_l = l_sum > 0.f ? 1.f / l_sum : 0.f;
-  if (it.part < 0) {
+  if (it.part < 0 && it.q_len == TILE) {
+    // Full tile: the slot's O goes through its Q region of shared memory (no
+    // MMA reads Q any more) in Q's swizzled layout, then out by TMA stores of
+    // one 64-column block of one head each: whole 128-byte rows instead of 16
+    // bytes per row and store.
+    const uint32_t stage = sbase + C::OFF_Q + slot * C::Q_BYTES + hp * TILE * 128 + row_local * 128;
+#pragma unroll
+    for (int c = 0; c < D / 32; ++c) {
+      uint32_t r[32];
+      ptx::tmem_ld32(tmem + C::COL_O + c * 32, r);
+      ptx::tmem_wait_ld();
+#pragma unroll
+      for (int q4 = 0; q4 < 4; ++q4) {
+        uint4 w;
+        w.x = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 0]) * inv_l, __uint_as_float(r[8 * q4 + 1]) * inv_l);
+        w.y = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 2]) * inv_l, __uint_as_float(r[8 * q4 + 3]) * inv_l);
+        w.z = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 4]) * inv_l, __uint_as_float(r[8 * q4 + 5]) * inv_l);
+        w.w = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 6]) * inv_l, __uint_as_float(r[8 * q4 + 7]) * inv_l);
+        // 16-byte chunk k of the row's 128-byte block kb sits at chunk k ^ (row & 7).
+        const int kb = c / 2, k = (c % 2) * 4 + q4;
+        const uint32_t addr = stage + kb * C::Q_BLOCK + ((k ^ (row_local & 7)) << 4);
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
+                     : "memory");
+      }
+    }
+    if (row_ok) L.lse[static_cast<int64_t>(head) * L.n_tok + qpos] = (m_used + __log2f(l_sum)) * kLn2;
+    ptx::fence_proxy_async_smem();
+    ptx::bar_sync(1 + slot, kRows);
+    if ((threadIdx.x & 127) == 0) {
+#pragma unroll
+      for (int h = 0; h < C::HP; ++h) {
+        if (slot * C::HP + h >= left) break;   // heads past the group's end are not stored
+#pragma unroll
+        for (int kb = 0; kb < C::KB; ++kb)
+          ptx::tma_store_3d(&L.tm_o, sbase + C::OFF_Q + slot * C::Q_BYTES + kb * C::Q_BLOCK + h * TILE * 128, kb * 64,
+                            it.head + slot * C::HP + h, it.q_start);
+      }
+      ptx::bulk_commit();
+      ptx::bulk_wait_read();   // the shared memory source must outlive the copy
+    }
+  } else if (it.part < 0) {
     uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(L.o) +
                                           (static_cast<int64_t>(qpos) * L.hq + head) * D);
 #pragma unroll
