@@ -11,9 +11,10 @@
 // over all row blocks in registers, closes each key over its 8 lanes, and the
 // block forms the frames (N_v divides 128) from the 128 token sums.
 //
-// evidence_finalize: head map (sum of a video's frames per head) and the
-// query-frame cue A_qf (sum over heads / (Hq * n_text)), both recomputed from
-// the frame map so that they accumulate over layers exactly as it does.
+// evidence_finalize: head map (sum of a video's frames per head; one warp per
+// video and head) and the query-frame cue A_qf (sum over heads / (Hq * n_text);
+// one thread per frame), both recomputed from the frame map so that they
+// accumulate over layers exactly as it does.
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -93,24 +94,37 @@ __global__ void __launch_bounds__(kWarps * 32) evidence_reduce_kernel(const __gr
   }
 }
 
-// Blocks [0, n_videos): head map of one video (one warp per head).
-// Blocks [n_videos, ...): A_qf, one thread per frame.
-__global__ void __launch_bounds__(256) evidence_finalize_kernel(const __grid_constant__ EvidenceLaunch L) {
-  if (blockIdx.x < static_cast<unsigned>(L.n_videos)) {
-    const VideoInfo vi = L.videos[blockIdx.x];
+// Blocks [0, n_videos * head_blocks): head map, one warp per (video, head),
+// four independent partial sums per lane. Blocks after those: A_qf, one
+// thread per frame.
+constexpr int kFinalizeWarps = 8;
+
+__global__ void __launch_bounds__(kFinalizeWarps * 32) evidence_finalize_kernel(const __grid_constant__ EvidenceLaunch L) {
+  const int head_blocks = (L.hq + kFinalizeWarps - 1) / kFinalizeWarps;
+  if (blockIdx.x < static_cast<unsigned>(L.n_videos * head_blocks)) {
+    const int b = blockIdx.x / head_blocks;
+    const int h = (blockIdx.x % head_blocks) * kFinalizeWarps + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (h >= L.hq) return;
+    const VideoInfo vi = L.videos[b];
     const int frames = vi.n_vis / L.tokens_per_frame;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int h = warp; h < L.hq; h += 8) {
-      const float* fr = L.frame + static_cast<int64_t>(h) * L.total_frames + vi.frame_off;
-      float s = 0.f;
-      for (int t = lane; t < frames; t += 32) s += fr[t];
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-      if (lane == 0) L.head[static_cast<int64_t>(blockIdx.x) * L.hq + h] = s;
+    const float* fr = L.frame + static_cast<int64_t>(h) * L.total_frames + vi.frame_off;
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    int t = lane;
+    for (; t + 96 < frames; t += 128) {
+      s0 += fr[t];
+      s1 += fr[t + 32];
+      s2 += fr[t + 64];
+      s3 += fr[t + 96];
     }
+    for (; t < frames; t += 32) s0 += fr[t];
+    float s = (s0 + s1) + (s2 + s3);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) L.head[static_cast<int64_t>(b) * L.hq + h] = s;
     return;
   }
-  const int t = (blockIdx.x - L.n_videos) * blockDim.x + threadIdx.x;
+  const int t = (blockIdx.x - L.n_videos * head_blocks) * blockDim.x + threadIdx.x;
   if (t >= L.total_frames) return;
   int lo = 0, hi = L.n_videos - 1;                 // video owning frame t
   while (lo < hi) {
@@ -119,9 +133,14 @@ __global__ void __launch_bounds__(256) evidence_finalize_kernel(const __grid_con
   }
   // (the last video whose frame offset is <= t always owns >= 1 frame)
   const VideoInfo vi = L.videos[lo];
-  float s = 0.f;
-  for (int h = 0; h < L.hq; ++h) s += L.frame[static_cast<int64_t>(h) * L.total_frames + t];
-  L.aqf[t] = vi.n_text > 0 ? s / (static_cast<float>(L.hq) * static_cast<float>(vi.n_text)) : 0.f;
+  float s0 = 0.f, s1 = 0.f;
+  int h = 0;
+  for (; h + 1 < L.hq; h += 2) {
+    s0 += L.frame[static_cast<int64_t>(h) * L.total_frames + t];
+    s1 += L.frame[static_cast<int64_t>(h + 1) * L.total_frames + t];
+  }
+  if (h < L.hq) s0 += L.frame[static_cast<int64_t>(h) * L.total_frames + t];
+  L.aqf[t] = vi.n_text > 0 ? (s0 + s1) / (static_cast<float>(L.hq) * static_cast<float>(vi.n_text)) : 0.f;
 }
 
 }  // namespace
@@ -133,9 +152,10 @@ cudaError_t launch_evidence(const EvidenceLaunch& L, cudaStream_t stream) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  const int aqf_blocks = (L.total_frames + 255) / 256;
-  if (L.n_videos + aqf_blocks > 0) {
-    evidence_finalize_kernel<<<L.n_videos + aqf_blocks, 256, 0, stream>>>(L);
+  const int head_blocks = (L.hq + kFinalizeWarps - 1) / kFinalizeWarps;
+  const int aqf_blocks = (L.total_frames + kFinalizeWarps * 32 - 1) / (kFinalizeWarps * 32);
+  if (L.n_videos * head_blocks + aqf_blocks > 0) {
+    evidence_finalize_kernel<<<L.n_videos * head_blocks + aqf_blocks, kFinalizeWarps * 32, 0, stream>>>(L);
     return cudaGetLastError();
   }
   return cudaSuccess;
