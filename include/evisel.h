@@ -171,6 +171,24 @@ int64_t evisel_workspace_bytes(const evisel_ws* ws);
 int evisel_probe_evidence_noalloc(const evisel_probe_args* args, float* tok, float* frame, float* head,
                                   float* aqf, int accumulate, void* stream, int* device_status);
 
+/* ---------------------------------------------------------------------------
+ * evisel_selftest_wait: failure detection check (no counterpart in the paper).
+ * Every wait in the library's kernels is bounded: it gives up after a time
+ * limit, records EVISEL_ETIMEOUT in a device status word and lets the kernel
+ * drain and exit, so that a stuck pipeline ends as an error the host can read
+ * instead of a hung GPU. This call runs that same bounded wait in a one-warp
+ * kernel on a barrier of its own, with a short limit:
+ *   - arrive = 0: nothing ever completes the barrier's phase, so the wait must
+ *     give up after about timeout_us microseconds: *device_status = EVISEL_ETIMEOUT;
+ *   - arrive = 1: the kernel completes the phase before waiting:
+ *     *device_status = EVISEL_OK.
+ * timeout_us: 1 .. 1000000. stream: cudaStream_t (NULL = legacy default).
+ * The call waits for `stream` and stores the kernel's status in *device_status
+ * (required). The device keeps working afterwards (nothing faults or traps).
+ * Returns EVISEL_OK, EVISEL_EINVAL (bad timeout or NULL device_status) or
+ * EVISEL_ECUDA. */
+int evisel_selftest_wait(int timeout_us, int arrive, void* stream, int* device_status);
+
 #ifdef __cplusplus
 }
 #endif

@@ -5,7 +5,8 @@ holds its sources (``csrc/``), the in-tree build and a thin ctypes binding with
 the same entry-point names. ``workloads`` draws the seeded synthetic inputs.
 """
 from ._binding import (  # noqa: F401
-    EviselError, Workspace, evisel_evidence_reduce, evisel_free, evisel_probe_attention, evisel_status, load,
+    EviselError, Workspace, evisel_evidence_reduce, evisel_free, evisel_probe_attention, evisel_probe_evidence_noalloc,
+    evisel_selftest_wait, evisel_status, load,
 )
 
 

@@ -79,6 +79,8 @@ def load(path: str = LIB_PATH):
     lib.evisel_probe_evidence_noalloc.argtypes = [ctypes.POINTER(ProbeArgs), vp, vp, vp, vp, i32, vp,
                                                   ctypes.POINTER(ctypes.c_int)]
     lib.evisel_probe_evidence_noalloc.restype = i32
+    lib.evisel_selftest_wait.argtypes = [i32, i32, vp, ctypes.POINTER(ctypes.c_int)]
+    lib.evisel_selftest_wait.restype = i32
     _lib = lib
     return lib
 
@@ -225,3 +227,13 @@ def evisel_probe_evidence_noalloc(q, k, v, cu_seqlens, n_vis, tokens_per_frame, 
                                              ctypes.byref(status) if wait_status else None))
     del keep
     return int(status.value) if wait_status else None
+
+
+def evisel_selftest_wait(timeout_us, arrive, stream=None):
+    """Runs the kernels' bounded wait on a barrier that is (arrive) or is not
+    completed; returns the device status word (0, or EVISEL_ETIMEOUT when the
+    wait gave up)."""
+    lib = load()
+    status = ctypes.c_int(1)
+    _check(lib.evisel_selftest_wait(int(timeout_us), int(bool(arrive)), _stream_handle(stream), ctypes.byref(status)))
+    return int(status.value)
