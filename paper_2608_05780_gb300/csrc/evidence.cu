@@ -26,7 +26,9 @@ namespace {
 constexpr int kChunk = 128;                        // visual keys per block
 constexpr int kWarps = kChunk / 32;                // one warp per 32 keys
 
-__global__ void __launch_bounds__(kWarps * 32) evidence_reduce_kernel(const __grid_constant__ EvidenceLaunch L) {
+// 16 blocks of 128 threads per SM (32 registers): the full 2,048 threads,
+// which the HBM stream needs (at 45 registers it ran 11 blocks and 26% slower).
+__global__ void __launch_bounds__(kWarps * 32, 16) evidence_reduce_kernel(const __grid_constant__ EvidenceLaunch L) {
   __shared__ float tok_s[kChunk];
   const int h = blockIdx.y;
   const EvChunk ck = L.chunks[blockIdx.x];
