@@ -28,6 +28,11 @@ Evidence (Sec. 3.2, "Evidence Decomposition"): with P from the text rows,
   A_qf[t]     = sum_h frame[h, t] / (Hq * n_text)   (average over the whole
                 query-token group and over heads; 0 for a video without query
                 tokens, a case the paper does not have)
+With P from the visual rows,
+  A_if[t, i, j] = (1 / Hq) sum_h P^h_(t N_v + i, t N_v + j) for j <= i, else 0:
+                the token-level causal attention inside frame t, head-averaged
+                (the intra-frame cue; P is the row's full softmax over all of
+                its allowed keys, so a frame row sums to its in-frame share).
 """
 from __future__ import annotations
 
@@ -35,7 +40,7 @@ import math
 
 import numpy as np
 
-__all__ = ["token_layout", "allowed_row", "probe_rows", "probe", "text_probabilities", "evidence"]
+__all__ = ["token_layout", "allowed_row", "probe_rows", "probe", "text_probabilities", "evidence", "intra_frame"]
 
 
 def token_layout(n_vis: int, n_text: int, tile: int):
@@ -179,3 +184,49 @@ def evidence(q, k, cu_seqlens, n_vis, tokens_per_frame, scale=None):
         if n_text > 0:      # a video without query tokens carries no query-frame evidence
             aqf[fr_off[b]:fr_off[b + 1]] = frame[:, fr_off[b]:fr_off[b + 1]].sum(axis=0) / (hq * n_text)
     return tok, frame, head, aqf
+
+
+def intra_frame(q, k, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, frames=None, scale=None,
+                chunk=512):
+    """Intra-frame cue A_if (Sec. 3.2, "Evidence Decomposition"): for frame t
+    (global index over the videos in order) the head-averaged causal attention
+    among its N_v visual tokens,
+        A_if[t, i, j] = (1 / Hq) sum_h P^h_(row i, key j),  j <= i,   0 above,
+    where P^h is the probe's probability (the row's softmax over all of its
+    allowed keys, Eq. 11). ``frames`` selects global frame indices (default:
+    all). Returns float64 [len(frames), N_v, N_v].
+    """
+    q = np.asarray(q); k = np.asarray(k)
+    hq, d = q.shape[1], q.shape[2]
+    hkv = k.shape[1]
+    gq = hq // hkv
+    npf = int(tokens_per_frame)
+    scale = 1.0 / math.sqrt(d) if not scale else float(scale)
+    n_vis = np.asarray(n_vis, dtype=np.int64)
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    n_frames = n_vis // npf
+    fr_off = np.concatenate([[0], np.cumsum(n_frames)])
+    frames = np.arange(int(fr_off[-1])) if frames is None else np.asarray(frames, dtype=np.int64)
+    retained = _video_csr_rows(cu, n_vis, tile, row_ptr, col_idx)
+    out = np.zeros((frames.size, npf, npf))
+    video_of = np.searchsorted(fr_off, frames, side="right") - 1
+    for b in np.unique(video_of):
+        sel = np.nonzero(video_of == b)[0]
+        s0, s1 = int(cu[b]), int(cu[b + 1])
+        nv = int(n_vis[b])
+        is_text, tile_id = token_layout(nv, s1 - s0 - nv, tile)
+        kb = k[s0:s1].astype(np.float64)
+        # the frames' rows, as local positions
+        local = ((frames[sel] - fr_off[b])[:, None] * npf + np.arange(npf)[None, :]).reshape(-1)
+        for c0 in range(0, local.size, chunk):
+            part = local[c0:c0 + chunk]
+            allowed = np.stack([allowed_row(int(p), is_text, tile_id, retained[b]) for p in part])
+            for h in range(hq):
+                _, _, p = _attend(q[s0 + part, h, :].astype(np.float64), kb[:, h // gq, :],
+                                  np.zeros((s1 - s0, 1)), allowed, scale)
+                for r, pos in enumerate(part):
+                    f = int(pos) // npf          # frame (video-local) of this row
+                    i = int(pos) % npf
+                    slot = sel[int(np.nonzero((frames[sel] - fr_off[b]) == f)[0][0])]
+                    out[slot, i, :] += p[r, f * npf:(f + 1) * npf] / hq
+    return out

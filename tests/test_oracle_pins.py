@@ -12,6 +12,7 @@ Each test names the pin it realises:
   O8  reductions: frame, head, A_qf from tok
   O9  planted frames rank top on the head-summed frame map
   O10 linearity of O in V
+  F1-F4 the intra-frame cue A_if (closed form, dense weights, brute force, structure)
 """
 import json
 import math
@@ -338,3 +339,103 @@ def test_pins_catch_planted_mistakes(monkeypatch):
     o, _ = op.probe(q, k, v, np.array([0, n]), np.array([4]), 2, np.array(g["row_ptr"]),
                     np.array(g["col_idx"]), scale=1.0)
     assert not np.allclose(o[:, 0, 0], g["expected_o"])
+
+
+# ---------------------------------------------------------------- intra-frame cue A_if
+# Pins of oracle.intra_frame (Sec. 3.2, "Evidence Decomposition"):
+#   F1  closed form for constant keys: P = 1/|allowed(row)| on j <= i
+#   F2  all-tiles mask: the diagonal frame blocks of dense causal attention
+#       weights (torch softmax over masked logits, float64), head-averaged
+#   F3  brute force, pure-Python loops, random masks, varlen
+#   F4  structure: zero above the diagonal; a video's first frame is
+#       row-stochastic (its rows see only their own frame); rows sum to <= 1
+def test_F1_intra_frame_constant_keys():
+    rng = np.random.default_rng(21)
+    n_vis, n_text, tile, d, npf, window = 24, 5, 8, 8, 4, 2
+    n = n_vis + n_text
+    cfg = wl.ProbeConfig("t", (n_vis // npf,), npf, (n_text,), 2, 1, d, tile, window)
+    row_ptr, col_idx = wl.build_mask(cfg)
+    q = rng.standard_normal((n, 2, d))
+    k = np.broadcast_to(rng.standard_normal(d), (n, 1, d)).copy()
+    a = oracle.intra_frame(q, k, [0, n], [n_vis], npf, tile, row_ptr, col_idx, scale=0.3)
+    for t in range(n_vis // npf):
+        for i in range(npf):
+            p = t * npf + i
+            cnt = _allowed_count_sink_window(p, n_vis, tile, window)
+            for j in range(npf):
+                want = 1.0 / cnt if j <= i else 0.0
+                assert abs(a[t, i, j] - want) < 1e-13, (t, i, j)
+
+
+def test_F2_intra_frame_all_tiles_equals_dense_causal_weights():
+    torch = pytest.importorskip("torch")
+    c = _random_case(23, videos=((12, 6), (8, 4)), density=1.0, tile=4, npf=4)
+    a = oracle.intra_frame(c["q"], c["k"], c["cu"], c["n_vis"], 4, c["tile"], c["row_ptr"], c["col_idx"])
+    hq, hkv, d = c["q"].shape[1], c["k"].shape[1], c["q"].shape[2]
+    f = 0
+    for b in range(2):
+        s0, s1, nv = int(c["cu"][b]), int(c["cu"][b + 1]), int(c["n_vis"][b])
+        qt = torch.from_numpy(c["q"][s0:s1].astype(np.float64)).transpose(0, 1)
+        kt = torch.from_numpy(c["k"][s0:s1].astype(np.float64)).transpose(0, 1).repeat_interleave(hq // hkv, 0)
+        logits = qt @ kt.transpose(1, 2) / math.sqrt(d)
+        n = s1 - s0
+        logits = logits.masked_fill(torch.triu(torch.ones(n, n, dtype=torch.bool), 1), float("-inf"))
+        w = torch.softmax(logits, dim=-1).mean(dim=0).numpy()        # head-averaged weights
+        for t in range(nv // 4):
+            np.testing.assert_allclose(a[f], w[4 * t:4 * t + 4, 4 * t:4 * t + 4], atol=1e-13)
+            f += 1
+
+
+@pytest.mark.parametrize("seed,tile,npf", [(24, 4, 2), (25, 8, 4)])
+def test_F3_intra_frame_brute_force(seed, tile, npf):
+    c = _random_case(seed, videos=((8, 3), (16, 5)), tile=tile, npf=npf, d=5)
+    a = oracle.intra_frame(c["q"], c["k"], c["cu"], c["n_vis"], npf, tile, c["row_ptr"], c["col_idx"])
+    _, lb = _brute(c, 1.0 / math.sqrt(5))
+    q, k = c["q"], c["k"]
+    hq, hkv = q.shape[1], k.shape[1]
+    f = 0
+    for b in range(2):
+        s0, nv = int(c["cu"][b]), int(c["n_vis"][b])
+        for t in range(nv // npf):
+            for i in range(npf):
+                row = s0 + t * npf + i
+                for j in range(npf):
+                    key = s0 + t * npf + j
+                    acc = 0.0
+                    if j <= i:     # the diagonal tile is always kept
+                        for h in range(hq):
+                            x = sum(float(q[row, h, e]) * float(k[key, h * hkv // hq, e]) for e in range(5))
+                            acc += math.exp(x / math.sqrt(5) - lb[h][row]) / hq
+                    assert abs(a[f, i, j] - acc) < 1e-12
+            f += 1
+
+
+def test_F4_intra_frame_structure():
+    c = _random_case(26, videos=((16, 4), (12, 5)), tile=8, npf=4, sharp=True)
+    a = oracle.intra_frame(c["q"], c["k"], c["cu"], c["n_vis"], 4, c["tile"], c["row_ptr"], c["col_idx"])
+    assert np.all(np.triu(a, 1) == 0.0)
+    assert np.all(a.sum(axis=2) <= 1.0 + 1e-12)
+    np.testing.assert_allclose(a[0].sum(axis=1), 1.0, atol=1e-12)          # video 0, frame 0
+    np.testing.assert_allclose(a[4].sum(axis=1), 1.0, atol=1e-12)          # video 1, frame 0
+    # a frame selection returns the same rows
+    sel = oracle.intra_frame(c["q"], c["k"], c["cu"], c["n_vis"], 4, c["tile"], c["row_ptr"], c["col_idx"],
+                             frames=[6, 1])
+    np.testing.assert_array_equal(sel, a[[6, 1]])
+
+
+def test_F1_catches_a_frame_local_softmax(monkeypatch):
+    """Planted mistake: normalising inside the frame instead of over the row's allowed keys."""
+    import oracle.attention as op
+    good = op._attend
+    npf = 4                                            # the frame size test_F1 uses
+
+    def frame_local(qh, kh, vh, allowed, scale):
+        o, lse, p = good(qh, kh, vh, allowed, scale)
+        out = np.zeros_like(p)
+        for r in range(p.shape[0]):
+            f0 = (np.nonzero(p[r])[0].max() // npf) * npf   # the row's own frame (its last allowed key is itself)
+            out[r, f0:f0 + npf] = p[r, f0:f0 + npf] / p[r, f0:f0 + npf].sum()
+        return o, lse, out
+    monkeypatch.setattr(op, "_attend", frame_local)
+    with pytest.raises(AssertionError):
+        test_F1_intra_frame_constant_keys()
