@@ -331,6 +331,28 @@ def bench_ours(args, cfg):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / args.steps
+
+    # The intra-frame cue A_if (a row beyond the probe step), timed on its own
+    # after the probe whose LSE it reads: HBM-bound (Q, K and LSE of the visual
+    # rows in, A_if out), with the diagonal logits recomputed on the tensor cores.
+    npf = cfg.tokens_per_frame
+    aif = torch.zeros((frames, npf, npf), device="cuda")
+
+    def intra_frame():
+        ev.evisel_intra_frame_evidence(q, k, v, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, probe.row_ptr,
+                                       probe.col_idx, o, lse, ws, aif=aif)
+
+    for _ in range(max(1, args.warmup)):
+        intra_frame()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        intra_frame()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if_ms = e0.elapsed_time(e1) / args.steps
+    if_bytes = total_vis * (hq * d * 2 + k.shape[1] * d * 2 + hq * 4) + frames * npf * npf * 4
+    if_flop = 2.0 * d * 128 * 128 * hq * sum(-(-int(nv) // 128) for nv in probe.n_vis)
     status = ev.evisel_status(ws)
     ws.free()
     if status != 0:
@@ -353,6 +375,9 @@ def bench_ours(args, cfg):
                              "traffic": _traffic(cfg.name),
                              "kernel": "probe_attn (evisel_probe_attention: probe_attn_kernel + attn_combine)",
                              "peak_source": f"{peaks['source']} bf16 burst"},
+                "intra_frame": {"ms": if_ms, "gbs": if_bytes / (if_ms * 1e-3) / 1e9,
+                                "frac_of_hbm": if_bytes / (if_ms * 1e-3) / 1e9 / peaks["hbm"], "bytes": if_bytes,
+                                "tflops": if_flop / (if_ms * 1e-3) / 1e12},
                 "e2e": {"value": world * st["flop"] / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
                         "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
                 "gpu_launches": args.steps * (4 if _has_combine(probe) else 3),

@@ -172,6 +172,30 @@ int evisel_probe_evidence_noalloc(const evisel_probe_args* args, float* tok, flo
                                   float* aqf, int accumulate, void* stream, int* device_status);
 
 /* ---------------------------------------------------------------------------
+ * evisel_intra_frame_evidence: the intra-frame cue A_if of Sec. 3.2
+ * ("Evidence Decomposition"): for every frame t (over the videos in order),
+ * the head-averaged token-level causal attention among its N_v visual tokens,
+ *     A_if[t, i, j] = (1 / hq) sum_h exp(s^h_ij - LSE^h_i),  j <= i,  0 above,
+ * with s = scale q_i k_j (Eq. 8) recomputed from Q/K and LSE the row's
+ * normaliser saved by the probe (Eq. 11), so each frame row sums to the share
+ * of its attention that stays inside the frame. E_if, the selector's
+ * intra-frame input, is A_if flattened per timestamp (and stacked over layers
+ * by the caller).
+ *   args   the arguments of the evisel_probe_attention() call that ran on `ws`
+ *          (q, k, cu_seqlens_h, n_vis_h, tokens_per_frame, hq, hkv, head_dim,
+ *          softmax_scale; args->lse is that call's LSE output, read here);
+ *          o/v/mask are not read but must be valid as for the probe.
+ *   ws     the workspace of that probe (read only; not modified).
+ *   aif    device fp32 [sum_b T_b, N_v, N_v], T_b = n_vis_h[b] / N_v.
+ *   accumulate  0: overwrite aif; 1: add to it (sum over layers).
+ * Asynchronous on `stream` (cudaStream_t, NULL = legacy default). Device-side
+ * timeouts are reported through evisel_status(ws).
+ * Errors: EVISEL_EINVAL (NULL aif or args as for the probe), EVISEL_ESTATE (no
+ * probe has run on ws), EVISEL_ECUDA. */
+int evisel_intra_frame_evidence(const evisel_probe_args* args, const evisel_ws* ws, float* aif, int accumulate,
+                                void* stream);
+
+/* ---------------------------------------------------------------------------
  * evisel_selftest_wait: failure detection check (no counterpart in the paper).
  * Every wait in the library's kernels is bounded: it gives up after a time
  * limit, records EVISEL_ETIMEOUT in a device status word and lets the kernel

@@ -79,6 +79,8 @@ def load(path: str = LIB_PATH):
     lib.evisel_probe_evidence_noalloc.argtypes = [ctypes.POINTER(ProbeArgs), vp, vp, vp, vp, i32, vp,
                                                   ctypes.POINTER(ctypes.c_int)]
     lib.evisel_probe_evidence_noalloc.restype = i32
+    lib.evisel_intra_frame_evidence.argtypes = [ctypes.POINTER(ProbeArgs), vp, vp, i32, vp]
+    lib.evisel_intra_frame_evidence.restype = i32
     lib.evisel_selftest_wait.argtypes = [i32, i32, vp, ctypes.POINTER(ctypes.c_int)]
     lib.evisel_selftest_wait.restype = i32
     _lib = lib
@@ -237,3 +239,22 @@ def evisel_selftest_wait(timeout_us, arrive, stream=None):
     status = ctypes.c_int(1)
     _check(lib.evisel_selftest_wait(int(timeout_us), int(bool(arrive)), _stream_handle(stream), ctypes.byref(status)))
     return int(status.value)
+
+
+def evisel_intra_frame_evidence(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse, ws,
+                                aif=None, accumulate=False, softmax_scale=0.0, stream=None):
+    """Intra-frame cue A_if [sum T, N_v, N_v] (fp32) of the probe that ran on ``ws``
+    with these arguments (o and lse are that probe's outputs)."""
+    import torch
+    lib = load()
+    n_vis_np = np.asarray(n_vis, dtype=np.int64)
+    frames = int(np.sum(n_vis_np // int(tokens_per_frame)))
+    if aif is None:
+        aif = torch.zeros((frames, int(tokens_per_frame), int(tokens_per_frame)), dtype=torch.float32,
+                          device=q.device)
+    args, keep = make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
+                           softmax_scale)
+    _check(lib.evisel_intra_frame_evidence(ctypes.byref(args), ws.ptr, aif.data_ptr(), int(bool(accumulate)),
+                                           _stream_handle(stream)))
+    del keep
+    return aif

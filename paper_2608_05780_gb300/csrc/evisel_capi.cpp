@@ -549,6 +549,50 @@ int evisel_evidence_reduce(const evisel_ws* ws_c, float* tok, float* frame, floa
   return EVISEL_OK;
 }
 
+int evisel_intra_frame_evidence(const evisel_probe_args* args, const evisel_ws* ws_c, float* aif, int accumulate,
+                                void* stream_ptr) {
+  g_last_error.clear();
+  evisel_ws* ws = const_cast<evisel_ws*>(ws_c);
+  if (!ws) return fail(EVISEL_EINVAL, "workspace is NULL");
+  int rc = validate(args);
+  if (rc != EVISEL_OK) return rc;
+  if (!ws->probed || !ws->have_plan) return fail(EVISEL_ESTATE, "no probe has run on this workspace");
+  const Plan& P = ws->plan;
+  if (static_cast<int>(P.videos.size()) != args->num_videos)
+    return fail(EVISEL_EINVAL, "args do not match the probe that ran on this workspace");
+  if (P.total_frames > 0 && !aif) return fail(EVISEL_EINVAL, "aif is NULL");
+  int max_vis = 0;
+  for (const VideoInfo& v : P.videos) max_vis = std::max(max_vis, v.n_vis);
+  if (max_vis == 0) return EVISEL_OK;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
+  IntraFrameLaunch L;
+  std::memset(&L, 0, sizeof(L));
+  rc = encode_map(&L.tm_q, args->q, P.n_tok, args->hq, args->head_dim, 128);
+  if (rc == EVISEL_OK) rc = encode_map(&L.tm_k, args->k, P.n_tok, args->hkv, args->head_dim, 128);
+  if (rc != EVISEL_OK) return rc;
+  const float scale = args->softmax_scale > 0.f ? args->softmax_scale : 1.0f / std::sqrt(float(args->head_dim));
+  L.videos = ws->d_videos;
+  L.lse = args->lse;
+  L.aif = aif;
+  L.status = ws->status;
+  L.n_videos = static_cast<int>(P.videos.size());
+  L.max_vis = max_vis;
+  L.n_tok = P.n_tok;
+  L.hq = args->hq;
+  L.hkv = args->hkv;
+  L.head_dim = args->head_dim;
+  L.tokens_per_frame = args->tokens_per_frame;
+  L.scale_log2 = scale * 1.4426950408889634f;
+  L.accumulate = accumulate != 0;
+  if (ws->last_stream != stream) {
+    cudaError_t e = cudaStreamWaitEvent(stream, ws->stage_done, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+  }
+  cudaError_t e = launch_intra_frame(L, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "intra_frame launch");
+  return EVISEL_OK;
+}
+
 void evisel_free(evisel_ws* ws) {
   if (!ws) return;
   int prev = -1;

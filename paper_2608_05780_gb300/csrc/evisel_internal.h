@@ -117,6 +117,21 @@ struct EvidenceLaunch {
 };
 
 // Kernel launchers (defined in the .cu files).
+// Intra-frame cue kernel: one CTA per 128-token block of a video's visual rows.
+struct IntraFrameLaunch {
+  CUtensorMap tm_q, tm_k;           // 3-D maps {d, heads, tokens}, box {64, 1, 128}, 128B swizzle
+  const VideoInfo* videos;
+  const float* lse;                 // [hq, N] from the probe
+  float* aif;                       // [sum T, N_v, N_v]
+  int* status;
+  int n_videos;
+  int max_vis;                      // largest n_vis of the batch (grid.x = row blocks)
+  int n_tok, hq, hkv, head_dim, tokens_per_frame;
+  float scale_log2;                 // softmax_scale * log2(e)
+  int accumulate;
+};
+
+cudaError_t launch_intra_frame(const IntraFrameLaunch& L, cudaStream_t stream);
 cudaError_t launch_probe_attn(const ProbeLaunch& L, cudaStream_t stream);
 cudaError_t launch_attn_combine(const CombineLaunch& L, cudaStream_t stream);
 cudaError_t launch_evidence(const EvidenceLaunch& L, cudaStream_t stream);
