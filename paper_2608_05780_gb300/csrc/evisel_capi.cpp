@@ -46,7 +46,8 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 }
 
 // 3-D bf16 tensor [tokens, heads, d] viewed as {d, heads, tokens}; box {64, 1, rows}.
-int encode_map(CUtensorMap* map, const void* base, int n_tok, int heads, int d, int rows) {
+int encode_map(CUtensorMap* map, const void* base, int n_tok, int heads, int d, int rows,
+               CUtensorMapL2promotion promotion = CU_TENSOR_MAP_L2_PROMOTION_L2_256B) {
   auto enc = tensor_map_encoder();
   if (!enc) return fail(EVISEL_ECUDA, "cuTensorMapEncodeTiled unavailable from the driver");
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(heads),
@@ -55,7 +56,7 @@ int encode_map(CUtensorMap* map, const void* base, int n_tok, int heads, int d, 
   cuuint32_t box[3] = {64, 1, static_cast<cuuint32_t>(rows)};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, promotion,
                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(EVISEL_ECUDA, "cuTensorMapEncodeTiled failed: " + std::to_string(r));
   return EVISEL_OK;
@@ -561,14 +562,17 @@ int evisel_intra_frame_evidence(const evisel_probe_args* args, const evisel_ws* 
   if (static_cast<int>(P.videos.size()) != args->num_videos)
     return fail(EVISEL_EINVAL, "args do not match the probe that ran on this workspace");
   if (P.total_frames > 0 && !aif) return fail(EVISEL_EINVAL, "aif is NULL");
-  int max_vis = 0;
-  for (const VideoInfo& v : P.videos) max_vis = std::max(max_vis, v.n_vis);
-  if (max_vis == 0) return EVISEL_OK;
+  int total_blocks = 0;
+  for (const VideoInfo& v : P.videos) total_blocks += (v.n_vis + 127) / 128;
+  if (total_blocks == 0) return EVISEL_OK;
   cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
   IntraFrameLaunch L;
   std::memset(&L, 0, sizeof(L));
-  rc = encode_map(&L.tm_q, args->q, P.n_tok, args->hq, args->head_dim, 128);
-  if (rc == EVISEL_OK) rc = encode_map(&L.tm_k, args->k, P.n_tok, args->hkv, args->head_dim, 128);
+  // No L2 promotion: each Q row of a head is read once, by one CTA (measured
+  // faster than 256-byte promotion for this pass).
+  rc = encode_map(&L.tm_q, args->q, P.n_tok, args->hq, args->head_dim, 128, CU_TENSOR_MAP_L2_PROMOTION_NONE);
+  if (rc == EVISEL_OK)
+    rc = encode_map(&L.tm_k, args->k, P.n_tok, args->hkv, args->head_dim, 128, CU_TENSOR_MAP_L2_PROMOTION_NONE);
   if (rc != EVISEL_OK) return rc;
   const float scale = args->softmax_scale > 0.f ? args->softmax_scale : 1.0f / std::sqrt(float(args->head_dim));
   L.videos = ws->d_videos;
@@ -576,7 +580,7 @@ int evisel_intra_frame_evidence(const evisel_probe_args* args, const evisel_ws* 
   L.aif = aif;
   L.status = ws->status;
   L.n_videos = static_cast<int>(P.videos.size());
-  L.max_vis = max_vis;
+  L.total_blocks = total_blocks;
   L.n_tok = P.n_tok;
   L.hq = args->hq;
   L.hkv = args->hkv;
@@ -590,6 +594,7 @@ int evisel_intra_frame_evidence(const evisel_probe_args* args, const evisel_ws* 
   }
   cudaError_t e = launch_intra_frame(L, stream);
   if (e != cudaSuccess) return cuda_fail(e, "intra_frame launch");
+  ws->last_stream = stream;
   return EVISEL_OK;
 }
 

@@ -125,7 +125,7 @@ struct IntraFrameLaunch {
   float* aif;                       // [sum T, N_v, N_v]
   int* status;
   int n_videos;
-  int max_vis;                      // largest n_vis of the batch (grid.x = row blocks)
+  int total_blocks;                 // 128-row blocks over all videos' visual rows
   int n_tok, hq, hkv, head_dim, tokens_per_frame;
   float scale_log2;                 // softmax_scale * log2(e)
   int accumulate;

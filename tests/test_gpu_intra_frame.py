@@ -22,15 +22,14 @@ RTOL = 2e-3
 ATOL = 1e-6
 
 
-def _gpu_aif(ev, probe, accumulate_into=None):
+def _gpu_aif(ev, probe, out=None, accumulate=False):
     import torch
     cfg = probe.cfg
     q, k, v = to_device(probe)
     o, lse, ws = ev.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
                                            probe.row_ptr, probe.col_idx)
     aif = ev.evisel_intra_frame_evidence(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
-                                         probe.row_ptr, probe.col_idx, o, lse, ws, aif=accumulate_into,
-                                         accumulate=accumulate_into is not None)
+                                         probe.row_ptr, probe.col_idx, o, lse, ws, aif=out, accumulate=accumulate)
     torch.cuda.synchronize()
     assert ev.evisel_status(ws) == 0
     ws.free()
@@ -86,9 +85,37 @@ def test_intra_frame_edge_cases(cuda_lib, name):
     _check(_gpu_aif(cuda_lib, probe), _oracle_aif(probe), name)
 
 
-def test_intra_frame_accumulates(cuda_lib):
+def _probe(name):
+    if name in EDGE:
+        from test_gpu_parity import _custom
+        return _custom(**EDGE[name])
+    return wl.make_probe(wl.CONFIGS[name])
+
+
+@pytest.mark.parametrize("name", ["tiny", "npf64"])
+def test_intra_frame_accumulates(cuda_lib, name):
     import torch
-    probe = wl.make_probe(wl.CONFIGS["tiny"])
+    probe = _probe(name)
     want = _oracle_aif(probe)
     base = torch.full(want.shape, 0.25, dtype=torch.float32, device="cuda")
-    _check(_gpu_aif(cuda_lib, probe, accumulate_into=base), want + 0.25, "accumulate")
+    _check(_gpu_aif(cuda_lib, probe, out=base, accumulate=True), want + 0.25, f"accumulate {name}")
+
+
+@pytest.mark.parametrize("name", ["single", "npf64", "npf4"])
+def test_intra_frame_overwrites(cuda_lib, name):
+    """Without accumulate every entry is written, the zeros above the diagonal included."""
+    import torch
+    probe = _probe(name)
+    want = _oracle_aif(probe)
+    out = torch.full(want.shape, float("nan"), dtype=torch.float32, device="cuda")
+    _check(_gpu_aif(cuda_lib, probe, out=out), want, f"overwrite {name}")
+
+
+def test_intra_frame_many_videos(cuda_lib):
+    """40 packed videos of 0-9 frames (fewer 128-row blocks than SMs, empty videos between)."""
+    from test_gpu_parity import _custom
+    rng = np.random.default_rng(11)
+    frames = tuple(int(f) for f in rng.integers(0, 10, size=40))
+    n_text = tuple(int(t) for t in rng.integers(1, 40, size=40))
+    probe = _custom(frames=frames, n_text=n_text, hq=4, hkv=2, d=128, tile=128, window=2)
+    _check(_gpu_aif(cuda_lib, probe), _oracle_aif(probe), "many videos")
