@@ -11,10 +11,12 @@ Every function here follows the paper's statement of the probe:
   * the frame-aligned block partition, text tokens partitioned independently
     (Appendix "Detailed Sparse Prefilling", the paragraph after Eq. 6);
   * logits q k^T / sqrt(d) (Eq. 8) and row-wise normalisation (Eq. 11);
-  * head averaging, the query-frame cue A_qf and the intra-frame cue A_if
-    (Sec. 3.2, "Evidence Decomposition").
+  * head averaging, the query-frame cue A_qf, the intra-frame cue A_if and
+    the cross-frame cue A_ff with its timestamp-aligned E_ff (Sec. 3.2,
+    "Evidence Decomposition").
 Parity pins for each function live in ``tests/test_oracle_pins.py``.
 """
 from .attention import (  # noqa: F401
-    token_layout, allowed_row, probe_rows, probe, text_probabilities, evidence, intra_frame,
+    token_layout, allowed_row, probe_rows, probe, text_probabilities, evidence, intra_frame, frame_mass_rows,
+    cross_frame, e_ff,
 )

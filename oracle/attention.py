@@ -33,6 +33,13 @@ With P from the visual rows,
                 the token-level causal attention inside frame t, head-averaged
                 (the intra-frame cue; P is the row's full softmax over all of
                 its allowed keys, so a frame row sums to its in-frame share).
+  A_ff[a-1, b]  = (1 / (N_v Hq)) sum_h sum_{i in frame a} sum_{j in frame b} P^h_ij
+                for the frames b < a of one video (the cross-frame cue: the
+                attention frame a gives to frame b, averaged over a's rows and
+                over heads), an array [(T-1), (T-1)] per video, 0 for b >= a
+  E_ff[t]       = ( sum_{b<t} A_ff[t-1, b] + sum_{a>t} A_ff[a-1, t] ) / 2: the
+                attention frame t gives to earlier frames and the attention it
+                receives from later ones, averaged (timestamp-aligned).
 """
 from __future__ import annotations
 
@@ -230,3 +237,91 @@ def intra_frame(q, k, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_id
                     slot = sel[int(np.nonzero((frames[sel] - fr_off[b]) == f)[0][0])]
                     out[slot, i, :] += p[r, f * npf:(f + 1) * npf] / hq
     return out
+
+
+def frame_mass_rows(q, k, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, frames, scale=None,
+                    chunk=512):
+    """For each global frame index a in ``frames``: the attention its visual
+    rows give to every frame b of the same video, averaged over the frame's
+    N_v rows and over heads,
+        M[a, b] = (1 / (N_v Hq)) sum_h sum_{i in a} sum_{j in b} P^h_ij,
+    with P the probe's probability (Eq. 11; the row's softmax over all of its
+    allowed keys). Returns a list of float64 vectors, one of length T_video
+    per requested frame (entries b > a are 0 by causality; b = a is the
+    in-frame share)."""
+    q = np.asarray(q); k = np.asarray(k)
+    hq, d = q.shape[1], q.shape[2]
+    hkv = k.shape[1]
+    gq = hq // hkv
+    npf = int(tokens_per_frame)
+    scale = 1.0 / math.sqrt(d) if not scale else float(scale)
+    n_vis = np.asarray(n_vis, dtype=np.int64)
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    n_frames = n_vis // npf
+    fr_off = np.concatenate([[0], np.cumsum(n_frames)])
+    frames = np.asarray(frames, dtype=np.int64)
+    retained = _video_csr_rows(cu, n_vis, tile, row_ptr, col_idx)
+    video_of = np.searchsorted(fr_off, frames, side="right") - 1
+    out = [np.zeros(int(n_frames[b])) for b in video_of]
+    for b in np.unique(video_of):
+        sel = np.nonzero(video_of == b)[0]
+        s0, s1 = int(cu[b]), int(cu[b + 1])
+        nv = int(n_vis[b])
+        tb = int(n_frames[b])
+        is_text, tile_id = token_layout(nv, s1 - s0 - nv, tile)
+        kb = k[s0:s1].astype(np.float64)
+        local = ((frames[sel] - fr_off[b])[:, None] * npf + np.arange(npf)[None, :]).reshape(-1)
+        slot_of_frame = {int(frames[i] - fr_off[b]): int(i) for i in sel}
+        for c0 in range(0, local.size, chunk):
+            part = local[c0:c0 + chunk]
+            allowed = np.stack([allowed_row(int(p), is_text, tile_id, retained[b]) for p in part])
+            for h in range(hq):
+                _, _, p = _attend(q[s0 + part, h, :].astype(np.float64), kb[:, h // gq, :],
+                                  np.zeros((s1 - s0, 1)), allowed, scale)
+                # mass of each row on each frame b' of the video (visual keys only)
+                per_frame = p[:, :tb * npf].reshape(len(part), tb, npf).sum(axis=2)
+                for r, pos in enumerate(part):
+                    out[slot_of_frame[int(pos) // npf]] += per_frame[r] / (npf * hq)
+    return out
+
+
+def cross_frame(q, k, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, scale=None, chunk=512):
+    """Cross-frame cue A_ff and its timestamp-aligned evidence E_ff (Sec. 3.2,
+    "Evidence Decomposition").
+
+    Returns (aff, eff): ``aff`` a list over videos of float64 [(T-1), (T-1)]
+    arrays with aff[a-1, b] = M[a, b] for b < a (M from ``frame_mass_rows``)
+    and 0 elsewhere; ``eff`` float64 [sum T] in video order, from ``e_ff``."""
+    n_vis = np.asarray(n_vis, dtype=np.int64)
+    npf = int(tokens_per_frame)
+    n_frames = n_vis // npf
+    fr_off = np.concatenate([[0], np.cumsum(n_frames)])
+    aff = []
+    for b in range(len(n_vis)):
+        tb = int(n_frames[b])
+        a_b = np.zeros((max(tb - 1, 0), max(tb - 1, 0)))
+        if tb > 1:
+            rows = frame_mass_rows(q, k, cu_seqlens, n_vis, npf, tile, row_ptr, col_idx,
+                                   np.arange(fr_off[b] + 1, fr_off[b] + tb), scale=scale, chunk=chunk)
+            for a in range(1, tb):
+                a_b[a - 1, :a] = rows[a - 1][:a]
+        aff.append(a_b)
+    return aff, e_ff(aff, n_frames)
+
+
+def e_ff(aff, n_frames):
+    """E_ff from A_ff: for frame t of a video with T frames,
+        E_ff[t] = ( sum_{b<t} A_ff[t-1, b] + sum_{a>t} A_ff[a-1, t] ) / 2
+    (the attention t gives to earlier frames, row t-1 of A_ff, and the
+    attention it receives from later frames, column t); an empty side is an
+    empty sum. Returns float64 [sum T]."""
+    out = []
+    for a_b, tb in zip(aff, n_frames):
+        tb = int(tb)
+        e = np.zeros(tb)
+        for t in range(tb):
+            give = a_b[t - 1, :t].sum() if t >= 1 else 0.0
+            recv = a_b[t:, t].sum() if t <= tb - 2 else 0.0     # rows a-1 = t .. T-2, i.e. frames a = t+1 .. T-1
+            e[t] = 0.5 * (give + recv)
+        out.append(e)
+    return np.concatenate(out) if out else np.zeros(0)

@@ -13,6 +13,8 @@ Each test names the pin it realises:
   O9  planted frames rank top on the head-summed frame map
   O10 linearity of O in V
   F1-F4 the intra-frame cue A_if (closed form, dense weights, brute force, structure)
+  G1-G5 the cross-frame cue A_ff and E_ff (closed form, mass balance with A_if, brute force,
+        dense weights, a hand-worked E_ff)
 """
 import json
 import math
@@ -439,3 +441,149 @@ def test_F1_catches_a_frame_local_softmax(monkeypatch):
     monkeypatch.setattr(op, "_attend", frame_local)
     with pytest.raises(AssertionError):
         test_F1_intra_frame_constant_keys()
+
+
+# ---------------------------------------------------------------- cross-frame cue A_ff, E_ff
+# Pins of oracle.frame_mass_rows / cross_frame / e_ff (Sec. 3.2, "Evidence
+# Decomposition"):
+#   G1  closed form for constant keys: A_ff[a-1, b] = mean over a's rows of
+#       |allowed(i) within frame b| / |allowed(i)|, counted from the tile rules
+#   G2  mass balance with the separately pinned A_if: for every frame,
+#       sum_b A_ff[a-1, b] + (1/N_v) sum_ij A_if[a, i, j] = 1 (a row's
+#       probabilities over its earlier frames and its own frame sum to one)
+#   G3  brute force, pure-Python loops, random masks, varlen
+#   G4  all-tiles mask: frame-block means of dense causal attention weights
+#       (torch softmax over masked logits, float64), head-averaged
+#   G5  E_ff on a hand-worked 3-frame example
+def test_G1_cross_frame_constant_keys():
+    rng = np.random.default_rng(31)
+    n_vis, n_text, tile, d, npf, window = 32, 5, 8, 8, 4, 2
+    n = n_vis + n_text
+    cfg = wl.ProbeConfig("t", (n_vis // npf,), npf, (n_text,), 2, 1, d, tile, window)
+    row_ptr, col_idx = wl.build_mask(cfg)
+    q = rng.standard_normal((n, 2, d))
+    k = np.broadcast_to(rng.standard_normal(d), (n, 1, d)).copy()
+    aff, _ = oracle.cross_frame(q, k, [0, n], [n_vis], npf, tile, row_ptr, col_idx, scale=0.3)
+    T = n_vis // npf
+    assert aff[0].shape == (T - 1, T - 1)
+    for a in range(1, T):
+        for b in range(T - 1):
+            want = 0.0
+            if b < a:
+                for i in range(npf):
+                    p = a * npf + i
+                    r = p // tile
+                    kept = {0} | set(range(max(0, r - window + 1), r + 1))
+                    inside = npf if (b * npf) // tile in kept else 0      # frame b lies in one tile, before row p
+                    want += inside / _allowed_count_sink_window(p, n_vis, tile, window) / npf
+            assert abs(aff[0][a - 1, b] - want) < 1e-13, (a, b)
+
+
+def test_G2_cross_frame_mass_balance():
+    c = _random_case(32, videos=((24, 5), (16, 7), (4, 3)), tile=8, npf=4, sharp=True)
+    args = (c["q"], c["k"], c["cu"], c["n_vis"], 4, c["tile"], c["row_ptr"], c["col_idx"])
+    aff, eff = oracle.cross_frame(*args)
+    aif = oracle.intra_frame(*args)
+    f = 0
+    for b, nv in enumerate(c["n_vis"]):
+        T = int(nv) // 4
+        for a in range(T):
+            earlier = aff[b][a - 1, :a].sum() if a >= 1 else 0.0
+            assert abs(earlier + aif[f].sum() / 4 - 1.0) < 1e-12, (b, a)
+            f += 1
+    assert eff.shape == (f,)
+    # the rows a frame selection returns are those of the full cue
+    rows = oracle.frame_mass_rows(*args, frames=[3, 7])
+    np.testing.assert_allclose(rows[0][:3], aff[0][2, :3], atol=0)
+    np.testing.assert_allclose(rows[1][:1], aff[1][0, :1], atol=0)
+
+
+@pytest.mark.parametrize("seed,tile,npf", [(33, 4, 2), (34, 8, 4)])
+def test_G3_cross_frame_brute_force(seed, tile, npf):
+    c = _random_case(seed, videos=((12, 3), (16, 5)), tile=tile, npf=npf, d=5)
+    aff, eff = oracle.cross_frame(c["q"], c["k"], c["cu"], c["n_vis"], npf, tile, c["row_ptr"], c["col_idx"])
+    _, lb = _brute(c, 1.0 / math.sqrt(5))
+    q, k, cu, n_vis = c["q"], c["k"], c["cu"], c["n_vis"]
+    hq, hkv = q.shape[1], k.shape[1]
+    row = 0
+    for b in range(2):
+        s0, nv = int(cu[b]), int(n_vis[b])
+        kept = []
+        for _ in range(-(-nv // tile)):
+            kept.append(set(int(x) for x in c["col_idx"][c["row_ptr"][row]:c["row_ptr"][row + 1]]))
+            row += 1
+        T = nv // npf
+        for a in range(1, T):
+            for fb in range(a):
+                acc = 0.0
+                for i in range(npf):
+                    pi = a * npf + i
+                    for j in range(npf):
+                        pj = fb * npf + j
+                        if pj // tile not in kept[pi // tile]:
+                            continue
+                        for h in range(hq):
+                            x = sum(float(q[s0 + pi, h, e]) * float(k[s0 + pj, h * hkv // hq, e]) for e in range(5))
+                            acc += math.exp(x / math.sqrt(5) - lb[h][s0 + pi]) / (npf * hq)
+                assert abs(aff[b][a - 1, fb] - acc) < 1e-12, (b, a, fb)
+            for fb in range(a, T - 1):
+                assert aff[b][a - 1, fb] == 0.0
+
+
+def test_G4_cross_frame_all_tiles_equals_dense_causal_weights():
+    torch = pytest.importorskip("torch")
+    c = _random_case(35, videos=((16, 6), (12, 4)), density=1.0, tile=4, npf=4)
+    aff, _ = oracle.cross_frame(c["q"], c["k"], c["cu"], c["n_vis"], 4, c["tile"], c["row_ptr"], c["col_idx"])
+    hq, hkv, d = c["q"].shape[1], c["k"].shape[1], c["q"].shape[2]
+    for b in range(2):
+        s0, s1, nv = int(c["cu"][b]), int(c["cu"][b + 1]), int(c["n_vis"][b])
+        qt = torch.from_numpy(c["q"][s0:s1].astype(np.float64)).transpose(0, 1)
+        kt = torch.from_numpy(c["k"][s0:s1].astype(np.float64)).transpose(0, 1).repeat_interleave(hq // hkv, 0)
+        logits = qt @ kt.transpose(1, 2) / math.sqrt(d)
+        n = s1 - s0
+        logits = logits.masked_fill(torch.triu(torch.ones(n, n, dtype=torch.bool), 1), float("-inf"))
+        w = torch.softmax(logits, dim=-1).mean(dim=0).numpy()
+        T = nv // 4
+        blocks = w[:nv, :nv].reshape(T, 4, T, 4).sum(axis=3).mean(axis=1)      # [a, b]: mean row mass
+        np.testing.assert_allclose(aff[b], np.tril(blocks[1:, :T - 1]), atol=1e-13)
+
+
+def test_G5_e_ff_hand_example():
+    # frames 0, 1, 2: A(1->0) = 0.2, A(2->0) = 0.3, A(2->1) = 0.4
+    aff = [np.array([[0.2, 0.0], [0.3, 0.4]])]
+    e = oracle.e_ff(aff, [3])
+    # E[0] = (0 + 0.2 + 0.3)/2, E[1] = (0.2 + 0.4)/2, E[2] = (0.3 + 0.4 + 0)/2
+    np.testing.assert_allclose(e, [0.25, 0.30, 0.35], atol=1e-15)
+    np.testing.assert_array_equal(oracle.e_ff([np.zeros((0, 0))], [1]), [0.0])
+
+
+def test_G5_catches_a_shifted_receive_column(monkeypatch):
+    """Planted mistake: the received attention read from column t - 1."""
+    import oracle.attention as op
+
+    def shifted(aff, n_frames):
+        out = []
+        for a_b, tb in zip(aff, n_frames):
+            e = np.zeros(int(tb))
+            for t in range(int(tb)):
+                give = a_b[t - 1, :t].sum() if t >= 1 else 0.0
+                recv = a_b[t:, t - 1].sum() if 1 <= t <= tb - 2 else 0.0
+                e[t] = 0.5 * (give + recv)
+            out.append(e)
+        return np.concatenate(out)
+    monkeypatch.setattr(op, "e_ff", shifted)
+    monkeypatch.setattr(oracle, "e_ff", shifted)
+    with pytest.raises(AssertionError):
+        test_G5_e_ff_hand_example()
+
+
+def test_G1_catches_a_block_mean_over_all_pairs(monkeypatch):
+    """Planted mistake: A_ff as the mean over all N_v x N_v entries (an extra 1/N_v)."""
+    import oracle.attention as op
+    good = op.frame_mass_rows
+
+    def per_entry(*a, **kw):
+        return [r / 4 for r in good(*a, **kw)]                 # N_v = 4 in test_G1
+    monkeypatch.setattr(op, "frame_mass_rows", per_entry)
+    with pytest.raises(AssertionError):
+        test_G1_cross_frame_constant_keys()
