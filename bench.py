@@ -358,6 +358,44 @@ def bench_ours(args, cfg):
     if status != 0:
         raise RuntimeError("device status reported an error")
 
+    # The cross-frame cue A_ff / E_ff (a row beyond the probe step): the probe
+    # run with its cross-frame partials (an extra output of the attention
+    # kernel), then the HBM-bound reduction of those partials, each timed on
+    # its own.
+    ws_cf = ev.Workspace()
+    pargs = (q, k, v, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, probe.row_ptr, probe.col_idx)
+    o_cf, lse_cf, ws_cf = ev.evisel_probe_attention(*pargs, ws=ws_cf, cross_frame=True)
+    t_frames = np.asarray(probe.n_vis) // npf
+    aff = torch.empty(int(np.sum(np.maximum(t_frames - 1, 0) ** 2)), device="cuda")
+    eff = torch.empty(frames, device="cuda")
+
+    def probe_cf():
+        ev.evisel_probe_attention(*pargs, ws=ws_cf, o=o_cf, lse=lse_cf, cross_frame=True)
+
+    def cross_frame():
+        ev.evisel_cross_frame_evidence(*pargs, o_cf, lse_cf, ws_cf, aff=aff, eff=eff)
+
+    def _time(fn):
+        for _ in range(max(1, args.warmup)):
+            fn()
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(args.steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / args.steps
+
+    pcf_ms = _time(probe_cf)
+    cf_ms = _time(cross_frame)
+    nnz = int(probe.row_ptr[-1])
+    fspill_bytes = hq * nnz * (cfg.tile // npf) * cfg.tile * 4
+    cf_bytes = fspill_bytes + hq * total_vis * 4 + aff.numel() * 4 + frames * 4
+    status = ev.evisel_status(ws_cf)
+    ws_cf.free()
+    if status != 0:
+        raise RuntimeError("device status reported an error")
+
     line = None
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
@@ -378,6 +416,10 @@ def bench_ours(args, cfg):
                 "intra_frame": {"ms": if_ms, "gbs": if_bytes / (if_ms * 1e-3) / 1e9,
                                 "frac_of_hbm": if_bytes / (if_ms * 1e-3) / 1e9 / peaks["hbm"], "bytes": if_bytes,
                                 "tflops": if_flop / (if_ms * 1e-3) / 1e12},
+                "cross_frame": {"probe_ms": pcf_ms, "probe_partials_bytes": fspill_bytes,
+                                "probe_overhead_ms": pcf_ms - attn_avg,
+                                "ms": cf_ms, "gbs": cf_bytes / (cf_ms * 1e-3) / 1e9,
+                                "frac_of_hbm": cf_bytes / (cf_ms * 1e-3) / 1e9 / peaks["hbm"], "bytes": cf_bytes},
                 "e2e": {"value": world * st["flop"] / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
                         "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
                 "gpu_launches": args.steps * (4 if _has_combine(probe) else 3),

@@ -87,6 +87,14 @@ typedef struct {
   void* o;                       /* device bf16 [N_tot, hq, d] (written)            */
   float* lse;                    /* device fp32 [hq, N_tot], natural log (written); must
                                     stay alive until evisel_evidence_reduce() ran  */
+  int32_t cross_frame;           /* 1: the probe also keeps, per visual row, kept kv
+                                    tile and key frame, the log-sum of the row's
+                                    attention on that frame, for
+                                    evisel_cross_frame_evidence() (needs
+                                    tokens_per_frame >= 16; workspace grows by
+                                    hq * nnz(mask) * tile * (tile / min(N_v, 64))
+                                    * 4 bytes).
+                                    0: not kept. Ignored by evisel_intra_frame_evidence. */
 } evisel_probe_args;
 
 /* Block-sparse causal GQA varlen attention (Eq. 1; Appendix Eq. 8 and Eq. 11
@@ -185,7 +193,8 @@ int evisel_probe_evidence_noalloc(const evisel_probe_args* args, float* tok, flo
  *          (q, k, cu_seqlens_h, n_vis_h, tokens_per_frame, hq, hkv, head_dim,
  *          softmax_scale; args->lse is that call's LSE output, read here);
  *          o/v/mask are not read but must be valid as for the probe.
- *   ws     the workspace of that probe (read only; not modified).
+ *   ws     the workspace of that probe (its plan is read; the call records
+ *          its stream there, so that evisel_status(ws) waits for it).
  *   aif    device fp32 [sum_b T_b, N_v, N_v], T_b = n_vis_h[b] / N_v.
  *   accumulate  0: overwrite aif; 1: add to it (sum over layers).
  * Asynchronous on `stream` (cudaStream_t, NULL = legacy default). Device-side
@@ -194,6 +203,33 @@ int evisel_probe_evidence_noalloc(const evisel_probe_args* args, float* tok, flo
  * probe has run on ws), EVISEL_ECUDA. */
 int evisel_intra_frame_evidence(const evisel_probe_args* args, const evisel_ws* ws, float* aif, int accumulate,
                                 void* stream);
+
+/* ---------------------------------------------------------------------------
+ * evisel_cross_frame_evidence: the cross-frame cue A_ff of Sec. 3.2 ("Evidence
+ * Decomposition") and its timestamp-aligned evidence E_ff. For frames b < a of
+ * one video,
+ *     A_ff[a-1, b] = (1 / (N_v hq)) sum_h sum_{i in frame a} sum_{j in frame b} P^h_ij,
+ * the attention frame a's visual rows give to frame b, averaged over a's rows
+ * and over heads (P the probe's probability, Eq. 11: pairs whose kv tile the
+ * mask does not keep are 0), and
+ *     E_ff[t] = ( sum_{b<t} A_ff[t-1, b] + sum_{a>t} A_ff[a-1, t] ) / 2,
+ * the attention frame t gives to earlier frames and the attention it receives
+ * from later ones, averaged.
+ *   args   the arguments of the evisel_probe_attention() call that ran on `ws`,
+ *          which must have had cross_frame = 1 (args->lse is read).
+ *   ws     that workspace (its plan and cross-frame partials are read; the call
+ *          records its stream there for evisel_status()).
+ *   aff    device fp32, the videos' [(T_b - 1), (T_b - 1)] row-major blocks back
+ *          to back in video order (sum_b (T_b - 1)^2 floats; entries b >= a are 0).
+ *   eff    device fp32 [sum_b T_b], or NULL to skip it. Always recomputed from
+ *          the resulting aff (so it follows aff's accumulation).
+ *   accumulate  0: overwrite aff (every entry is written); 1: add to it (sum
+ *          over layers).
+ * Asynchronous on `stream`. Errors: EVISEL_EINVAL (NULL aff when sum_b
+ * (T_b - 1)^2 > 0, args not matching the probe), EVISEL_ESTATE (no probe on
+ * ws, or it ran without cross_frame), EVISEL_ECUDA. */
+int evisel_cross_frame_evidence(const evisel_probe_args* args, evisel_ws* ws, float* aff, float* eff,
+                                int accumulate, void* stream);
 
 /* ---------------------------------------------------------------------------
  * evisel_selftest_wait: failure detection check (no counterpart in the paper).

@@ -44,6 +44,7 @@ class ProbeArgs(ctypes.Structure):
         ("mask_col_idx_h", ctypes.POINTER(ctypes.c_int32)),
         ("o", ctypes.c_void_p),
         ("lse", ctypes.c_void_p),
+        ("cross_frame", ctypes.c_int32),
     ]
 
 
@@ -81,6 +82,8 @@ def load(path: str = LIB_PATH):
     lib.evisel_probe_evidence_noalloc.restype = i32
     lib.evisel_intra_frame_evidence.argtypes = [ctypes.POINTER(ProbeArgs), vp, vp, i32, vp]
     lib.evisel_intra_frame_evidence.restype = i32
+    lib.evisel_cross_frame_evidence.argtypes = [ctypes.POINTER(ProbeArgs), vp, vp, vp, i32, vp]
+    lib.evisel_cross_frame_evidence.restype = i32
     lib.evisel_selftest_wait.argtypes = [i32, i32, vp, ctypes.POINTER(ctypes.c_int)]
     lib.evisel_selftest_wait.restype = i32
     _lib = lib
@@ -126,7 +129,7 @@ class Workspace:
 
 
 def make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
-              softmax_scale=0.0):
+              softmax_scale=0.0, cross_frame=False):
     """Fills the C struct; returns (struct, keepalive) - keepalive holds the host arrays."""
     cu, cu_p = _i32(cu_seqlens)
     nv, nv_p = _i32(n_vis)
@@ -146,12 +149,14 @@ def make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_i
     a.mask_row_ptr_h = rp_p
     a.mask_col_idx_h = ci_p
     a.o, a.lse = o.data_ptr(), lse.data_ptr()
+    a.cross_frame = int(bool(cross_frame))
     return a, (cu, nv, rp, ci)
 
 
 def evisel_probe_attention(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx,
-                           ws=None, o=None, lse=None, softmax_scale=0.0, stream=None):
+                           ws=None, o=None, lse=None, softmax_scale=0.0, stream=None, cross_frame=False):
     """Block-sparse GQA varlen probe attention. q/k/v: CUDA bf16 [N, H, d].
+    ``cross_frame`` also keeps the partials evisel_cross_frame_evidence reads.
 
     Returns (o [N, hq, d] bf16, lse [hq, N] fp32, ws).
     """
@@ -168,7 +173,7 @@ def evisel_probe_attention(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, r
     if ws is None:
         ws = Workspace()
     args, keep = make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
-                           softmax_scale)
+                           softmax_scale, cross_frame)
     _check(lib.evisel_probe_attention(ctypes.byref(args), _stream_handle(stream), ctypes.byref(ws.ptr)))
     del keep
     return o, lse, ws
@@ -258,3 +263,28 @@ def evisel_intra_frame_evidence(q, k, v, cu_seqlens, n_vis, tokens_per_frame, ti
                                            _stream_handle(stream)))
     del keep
     return aif
+
+
+def evisel_cross_frame_evidence(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse, ws,
+                                aff=None, eff=None, accumulate=False, softmax_scale=0.0, stream=None):
+    """Cross-frame cue A_ff (the videos' [(T-1), (T-1)] blocks back to back,
+    fp32) and E_ff [sum T] of the probe that ran on ``ws`` with cross_frame=True
+    and these arguments (o and lse are that probe's outputs).
+
+    Returns (aff, eff)."""
+    import torch
+    lib = load()
+    npf = int(tokens_per_frame)
+    t = np.asarray(n_vis, dtype=np.int64) // npf
+    n_aff = int(np.sum(np.maximum(t - 1, 0) ** 2))
+    if aff is None:
+        aff = torch.empty(n_aff, dtype=torch.float32, device=q.device)
+    if eff is None:
+        eff = torch.empty(int(np.sum(t)), dtype=torch.float32, device=q.device)
+    args, keep = make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
+                           softmax_scale, True)
+    _check(lib.evisel_cross_frame_evidence(ctypes.byref(args), ws.ptr, aff.data_ptr() if n_aff else None,
+                                           eff.data_ptr() if eff.numel() else None, int(bool(accumulate)),
+                                           _stream_handle(stream)))
+    del keep
+    return aff, eff

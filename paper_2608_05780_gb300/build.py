@@ -18,7 +18,8 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libevisel.so")
 
-SOURCES = ["probe_attn.cu", "attn_combine.cu", "evidence.cu", "evisel_capi.cpp", "evisel_noalloc.cu", "evisel_selftest.cu", "intra_frame.cu"]
+SOURCES = ["probe_attn.cu", "attn_combine.cu", "evidence.cu", "evisel_capi.cpp", "evisel_noalloc.cu", "evisel_selftest.cu", "intra_frame.cu",
+           "cross_frame.cu"]
 HEADERS = ["evisel_internal.h", "sm103_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",

@@ -74,6 +74,15 @@ struct Plan {
   int total_vis = 0;
   int total_frames = 0;
   int n_tok = 0;
+  // cross-frame partials (args->cross_frame)
+  bool cross_frame = false;
+  std::vector<VisRow> vrows;        // visual row tiles in mask order
+  std::vector<int64_t> aff_off;     // per video: float offset of its (T-1)^2 block of A_ff
+  int64_t aff_floats = 0;
+  int64_t fspill_floats = 0;
+  int nnz_vis = 0;                  // kept visual kv tiles (mask nonzeros)
+  int max_kv = 0;                   // longest mask row
+  int max_frames = 0;
 };
 
 int validate(const evisel_probe_args* a) {
@@ -92,6 +101,9 @@ int validate(const evisel_probe_args* a) {
     return fail(EVISEL_EUNSUPPORTED, "tokens_per_frame must be a power of two in [4, tile]");
   if (!(a->softmax_scale >= 0.f) || !std::isfinite(a->softmax_scale))
     return fail(EVISEL_EINVAL, "softmax_scale must be finite and >= 0");
+  if (a->cross_frame != 0 && a->cross_frame != 1) return fail(EVISEL_EINVAL, "cross_frame must be 0 or 1");
+  if (a->cross_frame && npf < 16)
+    return fail(EVISEL_EUNSUPPORTED, "cross-frame partials need tokens_per_frame >= 16");
   if (a->num_videos == 0) return EVISEL_OK;
   if (a->cu_seqlens_h[0] != 0) return fail(EVISEL_EINVAL, "cu_seqlens[0] must be 0");
   int64_t rows = 0;
@@ -190,6 +202,17 @@ void build_plan(const evisel_probe_args* a, Plan& P) {
       }
       const int cnt = static_cast<int>(P.kv.size()) - kv_begin;
       max_visual = std::max(max_visual, cnt);
+      if (a->cross_frame) {
+        VisRow vr{};
+        vr.q_start = v.vis_start + t * T;
+        vr.q_len = std::min(T, v.n_vis - t * T);
+        vr.video = b;
+        vr.row_tile = t;
+        vr.kv_begin = kv_begin;
+        vr.kv_count = cnt;
+        P.vrows.push_back(vr);
+        P.max_kv = std::max(P.max_kv, cnt);
+      }
       for (int h : head_blocks) {
         WorkItem it{};
         it.q_start = v.vis_start + t * T;
@@ -203,6 +226,21 @@ void build_plan(const evisel_probe_args* a, Plan& P) {
         items.push_back(it);
       }
     }
+  }
+
+  P.nnz_vis = static_cast<int>(P.kv.size());   // the visual kv lists come first, in mask order
+  if (a->cross_frame) {
+    P.cross_frame = true;
+    const int span = std::min(a->tokens_per_frame, 64);
+    P.fspill_floats = static_cast<int64_t>(hq) * P.nnz_vis * (T / span) * T;   // [hq, nnz, T / span, T]
+    int64_t off = 0;
+    for (int b = 0; b < a->num_videos; ++b) {
+      const int64_t tb = P.videos[b].n_vis / a->tokens_per_frame;
+      P.aff_off.push_back(off);
+      off += tb > 1 ? (tb - 1) * (tb - 1) : 0;
+      P.max_frames = std::max<int>(P.max_frames, static_cast<int>(tb));
+    }
+    P.aff_floats = off;
   }
 
   // Text row tiles: dense causal over the video, split into chunks no longer
@@ -313,6 +351,9 @@ struct evisel_ws {
   float* d_part_o = nullptr;
   float2* d_part_ml = nullptr;
   float* d_spill = nullptr;
+  VisRow* d_vrows = nullptr;
+  int64_t* d_aff_off = nullptr;
+  float* d_fspill = nullptr;
   // last probe, for the evidence pass
   bool probed = false;
   const float* lse = nullptr;
@@ -324,7 +365,7 @@ struct evisel_ws {
 namespace {
 
 std::vector<int32_t> plan_key(const evisel_probe_args* a) {
-  std::vector<int32_t> k = {a->num_videos, a->tokens_per_frame, a->hq, a->hkv, a->head_dim, a->tile};
+  std::vector<int32_t> k = {a->num_videos, a->tokens_per_frame, a->hq, a->hkv, a->head_dim, a->tile, a->cross_frame};
   for (int b = 0; b <= a->num_videos && a->num_videos > 0; ++b) k.push_back(a->cu_seqlens_h[b]);
   for (int b = 0; b < a->num_videos; ++b) k.push_back(a->n_vis_h[b]);
   int64_t rows = 0;
@@ -350,10 +391,13 @@ int install_plan(evisel_ws* ws, cudaStream_t stream) {
   const size_t o_videos = take(bytes_of(P.videos));
   const size_t o_groups = take(bytes_of(P.groups));
   const size_t o_chunks = take(bytes_of(P.chunks));
+  const size_t o_vrows = take(bytes_of(P.vrows));
+  const size_t o_aff_off = take(bytes_of(P.aff_off));
   const size_t meta_bytes = off;
   const size_t o_part_o = take(static_cast<size_t>(P.n_parts) * 128 * d * sizeof(float));
   const size_t o_part_ml = take(static_cast<size_t>(P.n_parts) * 128 * sizeof(float2));
   const size_t o_spill = take(static_cast<size_t>(P.spill_floats) * sizeof(float));
+  const size_t o_fspill = take(static_cast<size_t>(P.fspill_floats) * sizeof(float));
   const size_t total = std::max<size_t>(off, 256);
 
   if (total > ws->arena_bytes) {
@@ -392,6 +436,8 @@ int install_plan(evisel_ws* ws, cudaStream_t stream) {
   if (!P.videos.empty()) std::memcpy(h + o_videos, P.videos.data(), bytes_of(P.videos));
   if (!P.groups.empty()) std::memcpy(h + o_groups, P.groups.data(), bytes_of(P.groups));
   if (!P.chunks.empty()) std::memcpy(h + o_chunks, P.chunks.data(), bytes_of(P.chunks));
+  if (!P.vrows.empty()) std::memcpy(h + o_vrows, P.vrows.data(), bytes_of(P.vrows));
+  if (!P.aff_off.empty()) std::memcpy(h + o_aff_off, P.aff_off.data(), bytes_of(P.aff_off));
   char* base = static_cast<char*>(ws->arena);
   if (meta_bytes > 0) {
     cudaError_t e = cudaMemcpyAsync(base, h, meta_bytes, cudaMemcpyHostToDevice, stream);
@@ -407,6 +453,9 @@ int install_plan(evisel_ws* ws, cudaStream_t stream) {
   ws->d_part_o = reinterpret_cast<float*>(base + o_part_o);
   ws->d_part_ml = reinterpret_cast<float2*>(base + o_part_ml);
   ws->d_spill = reinterpret_cast<float*>(base + o_spill);
+  ws->d_vrows = reinterpret_cast<VisRow*>(base + o_vrows);
+  ws->d_aff_off = reinterpret_cast<int64_t*>(base + o_aff_off);
+  ws->d_fspill = reinterpret_cast<float*>(base + o_fspill);
   return EVISEL_OK;
 }
 
@@ -488,6 +537,11 @@ int evisel_probe_attention(const evisel_probe_args* args, void* stream_ptr, evis
     L.tile = args->tile;
     L.scale = scale;
     L.scale_log2 = scale * 1.4426950408889634f;
+    if (P.cross_frame && P.nnz_vis > 0) {
+      L.fspill = ws->d_fspill;
+      L.fs_nnz = P.nnz_vis;
+      L.fs_span = std::min(args->tokens_per_frame, 64);
+    }
     cudaError_t e = launch_probe_attn(L, stream);
     if (e != cudaSuccess) return cuda_fail(e, "probe_attn launch");
     if (!P.groups.empty()) {
@@ -594,6 +648,54 @@ int evisel_intra_frame_evidence(const evisel_probe_args* args, const evisel_ws* 
   }
   cudaError_t e = launch_intra_frame(L, stream);
   if (e != cudaSuccess) return cuda_fail(e, "intra_frame launch");
+  ws->last_stream = stream;
+  return EVISEL_OK;
+}
+
+int evisel_cross_frame_evidence(const evisel_probe_args* args, evisel_ws* ws, float* aff, float* eff,
+                                int accumulate, void* stream_ptr) {
+  g_last_error.clear();
+  if (!ws) return fail(EVISEL_EINVAL, "workspace is NULL");
+  int rc = validate(args);
+  if (rc != EVISEL_OK) return rc;
+  if (!ws->probed || !ws->have_plan) return fail(EVISEL_ESTATE, "no probe has run on this workspace");
+  const Plan& P = ws->plan;
+  if (!P.cross_frame) return fail(EVISEL_ESTATE, "the probe on this workspace ran without cross_frame");
+  if (static_cast<int>(P.videos.size()) != args->num_videos || plan_key(args) != ws->key)
+    return fail(EVISEL_EINVAL, "args do not match the probe that ran on this workspace");
+  if (P.aff_floats > 0 && !aff) return fail(EVISEL_EINVAL, "aff is NULL");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
+  if (ws->last_stream != stream) {
+    cudaError_t e = cudaStreamWaitEvent(stream, ws->stage_done, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+  }
+  if (!accumulate && P.aff_floats > 0) {
+    cudaError_t e = cudaMemsetAsync(aff, 0, static_cast<size_t>(P.aff_floats) * sizeof(float), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "A_ff clear");
+  }
+  CrossFrameLaunch L{};
+  L.rows = ws->d_vrows;
+  L.kv = ws->d_kv;
+  L.videos = ws->d_videos;
+  L.aff_off = ws->d_aff_off;
+  L.fspill = ws->d_fspill;
+  L.lse = args->lse;
+  L.aff = aff;
+  L.eff = P.total_frames > 0 ? eff : nullptr;
+  L.n_rows = P.aff_floats > 0 ? static_cast<int>(P.vrows.size()) : 0;
+  L.n_videos = static_cast<int>(P.videos.size());
+  L.max_frames = P.max_frames;
+  L.max_kv = P.max_kv;
+  L.nnz = P.nnz_vis;
+  L.fpt = args->tile / std::min(args->tokens_per_frame, 64);
+  L.spans_per_frame = args->tokens_per_frame / std::min(args->tokens_per_frame, 64);
+  L.tokens_per_frame = args->tokens_per_frame;
+  L.tile = args->tile;
+  L.n_tok = P.n_tok;
+  L.hq = args->hq;
+  L.accumulate = accumulate != 0;
+  cudaError_t e = launch_cross_frame(L, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cross_frame launch");
   ws->last_stream = stream;
   return EVISEL_OK;
 }

@@ -88,6 +88,12 @@ struct ProbeLaunch {
   int hq, hkv, head_dim, tile;
   float scale_log2;                 // softmax_scale * log2(e)
   float scale;                      // softmax_scale
+  // Cross-frame partials of the visual rows (null when not requested):
+  // [hq, fs_nnz, tile / fs_span, tile] fp32, fs_nnz = kept visual kv tiles
+  // (the mask's nonzeros, in mask order), fs_span = min(N_v, 64) keys per
+  // partial (a key frame is N_v / fs_span consecutive spans).
+  float* fspill;
+  int fs_nnz, fs_span;
 };
 
 struct CombineLaunch {
@@ -131,7 +137,37 @@ struct IntraFrameLaunch {
   int accumulate;
 };
 
+// One visual row tile of the mask, for the cross-frame reduction.
+struct VisRow {
+  int32_t q_start;    // global index of the tile's first token
+  int32_t q_len;      // rows (<= tile)
+  int32_t video;
+  int32_t row_tile;   // video-local tile index
+  int32_t kv_begin;   // its first kept tile: index into the mask nonzeros (and the KvTile list)
+  int32_t kv_count;
+  int32_t pad0, pad1;
+};
+static_assert(sizeof(VisRow) == 32, "VisRow is 32 bytes");
+
+struct CrossFrameLaunch {
+  const VisRow* rows;
+  const KvTile* kv;
+  const VideoInfo* videos;
+  const int64_t* aff_off;           // [videos] float offset of each video's (T-1)^2 block
+  const float* fspill;              // [hq, nnz, fpt, tile] from the probe (spans of tile / fpt keys)
+  const float* lse;                 // [hq, N]
+  float* aff;
+  float* eff;                       // may be null
+  int n_rows, n_videos, max_frames;
+  int max_kv;                       // longest kept-tile list of a row tile
+  int nnz, fpt, tokens_per_frame, tile;   // fpt: partial spans per tile
+  int spans_per_frame;              // N_v / span
+  int n_tok, hq;
+  int accumulate;
+};
+
 cudaError_t launch_intra_frame(const IntraFrameLaunch& L, cudaStream_t stream);
+cudaError_t launch_cross_frame(const CrossFrameLaunch& L, cudaStream_t stream);
 cudaError_t launch_probe_attn(const ProbeLaunch& L, cudaStream_t stream);
 cudaError_t launch_attn_combine(const CombineLaunch& L, cudaStream_t stream);
 cudaError_t launch_evidence(const EvidenceLaunch& L, cudaStream_t stream);

@@ -346,7 +346,7 @@ __device__ __forceinline__ void mma_issuer(const ProbeLaunch& L, const WorkItem&
   __syncwarp();
 }
 
-template <int TILE, int D, int NS>
+template <int TILE, int D, int NS, int FSW>
 __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const WorkItem& it, int slot, uint32_t sbase,
                                                  uint32_t tmem_base, volatile int* abort_flag) {
   using C = Cfg<TILE, D, NS>;
@@ -379,6 +379,18 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
       spill_row = L.spill + vi.spill_off + static_cast<int64_t>(head) * vi.n_vis * vi.text_pitch +
                   static_cast<int64_t>(r >> 5) * vi.n_vis * 32 + (r & 31);
     }
+  }
+
+  // Cross-frame partials (visual rows, when enabled): per kept kv tile and
+  // key frame f, m + log2(sum of the frame's P) in log2 units, so that the
+  // frame's share of the row's softmax is exp2(value - LSE log2 e).
+  // FSW = the key span of one partial, min(N_v, 64), in the instantiation that
+  // keeps them (0: not kept), so that the span ends are compile-time positions
+  // and the plain probe is unchanged.
+  float* fs_row = nullptr;
+  if constexpr (FSW > 0) {
+    if (it.text_row0 < 0 && row_ok)
+      fs_row = L.fspill + (static_cast<int64_t>(head) * L.fs_nnz + it.kv_begin) * (TILE / FSW) * TILE + row_local;
   }
 
   float m_used = -INFINITY;   // running max, log2 units
@@ -473,6 +485,11 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
     // the chunk's P is stored, and P of chunk h lands below chunk h + 1).
     const uint64_t negm2 = ptx::f2(-m_safe, -m_safe);
     uint64_t l2[4] = {0, 0, 0, 0};
+    [[maybe_unused]] float l_tile = 0.f;
+    [[maybe_unused]] float* fs_tile = nullptr;
+    if constexpr (FSW > 0) {
+      if (fs_row) fs_tile = fs_row + static_cast<int64_t>(j) * (TILE / FSW) * TILE;
+    }
 #pragma unroll
     for (int h = 0; h < TILE / 64; ++h) {
       float s[64];
@@ -500,10 +517,26 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
         const float p1 = ptx::ex2(x1);
         l2[e & 3] = ptx::add2(l2[e & 3], ptx::f2(p0, p1));
         pk[e] = ptx::pack_bf16x2(p0, p1);
+        if constexpr (FSW > 0) {
+          if ((h * 64 + 2 * e + 2) % FSW == 0) {      // the last keys of span (h * 64 + 2e + 2) / FSW - 1
+            float a0, a1, b0, b1, c0, c1, d0, d1;
+            ptx::unf2(l2[0], a0, a1);
+            ptx::unf2(l2[1], b0, b1);
+            ptx::unf2(l2[2], c0, c1);
+            ptx::unf2(l2[3], d0, d1);
+            const float fsum = ((a0 + a1) + (b0 + b1)) + ((c0 + c1) + (d0 + d1));
+            l_tile += fsum;
+            l2[0] = l2[1] = l2[2] = l2[3] = 0;
+            if (fs_tile)
+              __stcs(fs_tile + ((h * 64 + 2 * e + 2) / FSW - 1) * TILE, fsum > 0.f ? m_safe + __log2f(fsum) : -INFINITY);
+          }
+        }
       }
       ptx::tmem_st32(tS + h * 32, pk);
     }
-    {
+    if constexpr (FSW > 0) {
+      l_sum += l_tile;
+    } else {
       float a0, a1, b0, b1, c0, c1, d0, d1;
       ptx::unf2(l2[0], a0, a1);
       ptx::unf2(l2[1], b0, b1);
@@ -605,7 +638,7 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
   }
 }
 
-template <int TILE, int D, int NS>
+template <int TILE, int D, int NS, int FSW>
 __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_constant__ ProbeLaunch L) {
   using C = Cfg<TILE, D, NS>;
   extern __shared__ uint8_t smem_raw[];
@@ -640,7 +673,7 @@ __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_co
   } else if (warp == kWarpMma) {
     mma_issuer<TILE, D, NS>(L, it, sbase, tmem, abort_flag);
   } else {
-    softmax_epilogue<TILE, D, NS>(L, it, warp / 4, sbase, tmem, abort_flag);
+    softmax_epilogue<TILE, D, NS, FSW>(L, it, warp / 4, sbase, tmem, abort_flag);
   }
   ptx::tc_fence_before();
   __syncthreads();
@@ -650,11 +683,11 @@ __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_co
   }
 }
 
-template <int TILE, int D>
+template <int TILE, int D, int FSW>
 cudaError_t launch_cfg(const ProbeLaunch& L, cudaStream_t stream) {
   constexpr int NS = 2;
   using C = Cfg<TILE, D, NS>;
-  auto kern = probe_attn_kernel<TILE, D, NS>;
+  auto kern = probe_attn_kernel<TILE, D, NS, FSW>;
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
@@ -665,14 +698,28 @@ cudaError_t launch_cfg(const ProbeLaunch& L, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
+// The plain probe (fsw = 0) or the one that keeps cross-frame partials over
+// key spans of fsw tokens (16, 32 or 64).
+template <int TILE, int D>
+cudaError_t launch_fsw(const ProbeLaunch& L, int fsw, cudaStream_t stream) {
+  switch (fsw) {
+    case 0: return launch_cfg<TILE, D, 0>(L, stream);
+    case 16: return launch_cfg<TILE, D, 16>(L, stream);
+    case 32: return launch_cfg<TILE, D, 32>(L, stream);
+    case 64: return launch_cfg<TILE, D, 64>(L, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_probe_attn(const ProbeLaunch& L, cudaStream_t stream) {
   if (L.n_items == 0) return cudaSuccess;
-  if (L.tile == 128 && L.head_dim == 128) return launch_cfg<128, 128>(L, stream);
-  if (L.tile == 128 && L.head_dim == 64) return launch_cfg<128, 64>(L, stream);
-  if (L.tile == 64 && L.head_dim == 128) return launch_cfg<64, 128>(L, stream);
-  if (L.tile == 64 && L.head_dim == 64) return launch_cfg<64, 64>(L, stream);
+  const int fsw = L.fspill ? L.fs_span : 0;
+  if (L.tile == 128 && L.head_dim == 128) return launch_fsw<128, 128>(L, fsw, stream);
+  if (L.tile == 128 && L.head_dim == 64) return launch_fsw<128, 64>(L, fsw, stream);
+  if (L.tile == 64 && L.head_dim == 128) return launch_fsw<64, 128>(L, fsw, stream);
+  if (L.tile == 64 && L.head_dim == 64) return launch_fsw<64, 64>(L, fsw, stream);
   return cudaErrorInvalidValue;
 }
 

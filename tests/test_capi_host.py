@@ -66,6 +66,7 @@ def _args(**over):
     a.q, a.k, a.v, a.o, a.lse = p["q"], p["k"], p["v"], p["o"], p["lse"]
     a.mask_row_ptr_h = arr(p["row_ptr"])
     a.mask_col_idx_h = arr(p["col_idx"] or [0])
+    a.cross_frame = p.get("cross_frame", 0)
     return a, keep
 
 
@@ -93,6 +94,8 @@ def _args(**over):
     (dict(col_idx=[0, 0, 1, -1, 2, 2, 3]), -3),      # negative tile
     (dict(row_ptr=[0, 1, 1, 5, 7]), -3),             # empty row
     (dict(row_ptr=[1, 1, 3, 5, 7]), -3),
+    (dict(cross_frame=2), -1),
+    (dict(cross_frame=1, npf=8, n_vis=[256]), -2),   # cross-frame partials need N_v >= 16
 ])
 def test_validation_rejects(lib, over, code):
     a, keep = _args(**over)
@@ -110,6 +113,19 @@ def test_null_workspace_pointer(lib):
 
 def test_evidence_without_probe(lib):
     assert lib.evisel_evidence_reduce(None, None, None, None, None, 0, None) == -1
+
+
+def test_cross_frame_without_workspace(lib):
+    a, keep = _args(cross_frame=1)
+    assert lib.evisel_cross_frame_evidence(ctypes.byref(a), None, None, None, 0, None) == -1
+
+
+def test_noalloc_rejects_cross_frame(lib):
+    a, keep = _args(cross_frame=1)
+    st = ctypes.c_int(0)
+    rc = lib.evisel_probe_evidence_noalloc(ctypes.byref(a), ctypes.c_void_p(FAKE), ctypes.c_void_p(FAKE),
+                                           ctypes.c_void_p(FAKE), ctypes.c_void_p(FAKE), 0, None, ctypes.byref(st))
+    assert rc == -2, lib.evisel_last_error()
 
 
 def test_free_null_is_safe(lib):
