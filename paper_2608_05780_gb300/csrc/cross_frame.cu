@@ -10,15 +10,18 @@
 // there. The span's share of the row's softmax (Eq. 11) is then
 // 2^(value - LSE_i log2 e), with LSE the probe's final normaliser.
 //
-// cross_frame_pairs_kernel: one CTA per (visual row tile, 8 kept tiles), one
-// thread per row. A thread sums its row's shares over the heads, the CTA sums
-// them over the N_v rows of each query frame (shuffles, then a shared-memory
-// step for N_v > 32), and the first row of the frame writes A_ff[a-1, b]. A
-// frame pair (a, b) belongs to exactly one (row tile, kept tile), so every
-// entry has one writer and a fixed summation order (deterministic).
+// cross_frame_pairs_kernel: one CTA per (visual row tile, 16 consecutive
+// (kept tile, span) units), one thread per row. A thread sums its row's
+// shares over the heads for all 16 units at once (16 independent loads per
+// head), the CTA sums them over the N_v rows of each query frame (shuffles,
+// then a shared-memory step for N_v > 32), and the first row of the frame
+// adds the spans of each key frame and writes A_ff[a-1, b]. A frame pair
+// (a, b) belongs to exactly one (row tile, kept tile), so every entry has one
+// writer and a fixed summation order (deterministic).
 // e_ff_kernel: one CTA per (32 frames, video) forms E_ff from A_ff: the
-// received attention by column sums (8 warps over the rows, coalesced), the
-// given attention by row sums (a warp per row), partials added in a fixed order.
+// received attention by column sums (32 warps over the rows, coalesced), the
+// given attention by row sums (a warp per frame), partials added in a fixed
+// order.
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -28,67 +31,88 @@
 namespace evisel {
 namespace {
 
-constexpr int kKvPerCta = 8;
+constexpr int kUnits = 16;                       // (kept tile, key span) units per CTA
 constexpr unsigned kFull = 0xffffffffu;
 
 template <int TILE>
 __global__ void __launch_bounds__(TILE) cross_frame_pairs_kernel(const __grid_constant__ CrossFrameLaunch L) {
-  extern __shared__ float lse2[];                  // [hq][TILE]: each thread's own column
-  __shared__ float red[TILE / 32];
+  __shared__ float red[TILE / 32][kUnits];
   const VisRow R = L.rows[blockIdx.x];
-  const int k0 = blockIdx.y * kKvPerCta;
-  if (k0 >= R.kv_count) return;                    // uniform over the CTA
-  const int k1 = min(R.kv_count, k0 + kKvPerCta);
+  const int fpt = L.fpt;                           // spans per kv tile (1, 2, 4 or 8; divides kUnits)
+  const int u0 = blockIdx.y * kUnits;              // first unit: kept tile u0 / fpt, span u0 % fpt
+  if (u0 >= R.kv_count * fpt) return;              // uniform over the CTA
+  const int n_u = min(kUnits, R.kv_count * fpt - u0);
   const VideoInfo vi = L.videos[R.video];
-  const int npf = L.tokens_per_frame, fpt = L.fpt;
+  const int npf = L.tokens_per_frame, spf = L.spans_per_frame;
   const int T = vi.n_vis / npf;
   const int row = threadIdx.x, lane = row & 31, warp = row >> 5;
   const bool valid = row < R.q_len;
-  for (int h = 0; h < L.hq; ++h)
-    lse2[h * TILE + row] = valid ? L.lse[static_cast<int64_t>(h) * L.n_tok + R.q_start + row] * 1.4426950408889634f
-                                 : 0.f;
-  const int a = (R.row_tile * TILE + row) / npf;  // the row's frame (video-local)
-  const float inv_norm = 1.f / static_cast<float>(npf * L.hq);
-  const int64_t head_stride = static_cast<int64_t>(L.nnz) * fpt * TILE;
-  float* aff = L.aff + L.aff_off[R.video];
-  for (int k = k0; k < k1; ++k) {
-    const int p = R.kv_begin + k;
-    const int c_tile = (L.kv[p].start - vi.vis_start) / TILE;
-    const int spf = L.spans_per_frame;
-    float v = 0.f;
-    for (int f = 0; f < fpt; ++f) {
-      if (valid) {
-        const float* src = L.fspill + (static_cast<int64_t>(p) * fpt + f) * TILE + row;
-#pragma unroll 4
-        for (int h = 0; h < L.hq; ++h) v += ptx::ex2(__ldcs(src + h * head_stride) - lse2[h * TILE + row]);
-      }
-      if ((f + 1) % spf != 0) continue;            // the key frame has another span
-      const int b = (c_tile * fpt + f) / spf;      // key frame (video-local)
-      // Sum over the N_v rows of the query frame (aligned groups of threads).
-      const int w = npf < 32 ? npf : 32;
-      for (int off = w / 2; off > 0; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
-      if (npf > 32) {
-        if (lane == 0) red[warp] = v;
-        __syncthreads();
-        if (row % npf == 0) {
-          float t = 0.f;
-          for (int ww = warp; ww < warp + npf / 32; ++ww) t += red[ww];
-          v = t;
-        }
-        __syncthreads();
-      }
-      if (row % npf == 0 && b < a && a < T) {
-        float* dst = aff + static_cast<int64_t>(a - 1) * (T - 1) + b;
-        const float val = v * inv_norm;
-        *dst = L.accumulate ? *dst + val : val;
-      }
-      v = 0.f;
+  const int a = (R.row_tile * TILE + row) / npf;   // the row's frame (video-local)
+  // Units u0 .. u0 + 15 are consecutive spans of consecutive kept tiles: for a
+  // head they are one contiguous run of 16 x TILE floats.
+  float v[kUnits];
+#pragma unroll
+  for (int u = 0; u < kUnits; ++u) v[u] = 0.f;
+  if (valid) {
+    const float* src = L.fspill + (static_cast<int64_t>(R.kv_begin) * fpt + u0) * TILE + row;
+    const int64_t head_stride = static_cast<int64_t>(L.nnz) * fpt * TILE;
+    const float* lse = L.lse + R.q_start + row;
+    for (int h = 0; h < L.hq; ++h) {
+      const float m = __ldg(lse + static_cast<int64_t>(h) * L.n_tok) * 1.4426950408889634f;
+      const float* sh = src + h * head_stride;
+#pragma unroll
+      for (int u = 0; u < kUnits; ++u)
+        if (u < n_u) v[u] += ptx::ex2(__ldcs(sh + u * TILE) - m);
     }
+  }
+  // Spans -> key frames (spf consecutive units), then sums over the N_v rows
+  // of each query frame: shuffles inside a warp, shared memory across warps.
+  const int w = npf < 32 ? npf : 32;
+#pragma unroll
+  for (int u = 0; u < kUnits; ++u) {
+    float x = v[u];
+    for (int off = w / 2; off > 0; off >>= 1) x += __shfl_xor_sync(kFull, x, off);
+    v[u] = x;
+  }
+  if (npf > 32) {
+    if (lane == 0) {
+#pragma unroll
+      for (int u = 0; u < kUnits; ++u) red[warp][u] = v[u];
+    }
+    __syncthreads();
+    if (row % npf == 0) {
+#pragma unroll
+      for (int u = 0; u < kUnits; ++u) {
+        float t = 0.f;
+        for (int ww = warp; ww < warp + npf / 32; ++ww) t += red[ww][u];
+        v[u] = t;
+      }
+    }
+  }
+  if (row % npf != 0 || a >= T) return;
+  const float inv_norm = 1.f / static_cast<float>(npf * L.hq);
+  float* aff = L.aff + L.aff_off[R.video] + static_cast<int64_t>(a - 1) * (T - 1);
+  float fsum = 0.f;
+#pragma unroll
+  for (int u = 0; u < kUnits; ++u) {
+    if (u >= n_u) break;
+    fsum += v[u];
+    const int uu = u0 + u;                         // unit within the row's list
+    if ((uu % fpt + 1) % spf != 0) continue;       // the key frame has another span
+    const int c_tile = (L.kv[R.kv_begin + uu / fpt].start - vi.vis_start) / TILE;
+    const int b = (c_tile * fpt + uu % fpt) / spf; // key frame (video-local)
+    if (b < a) {
+      const float val = fsum * inv_norm;
+      aff[b] = L.accumulate ? aff[b] + val : val;
+    }
+    fsum = 0.f;
   }
 }
 
-__global__ void __launch_bounds__(256) e_ff_kernel(const __grid_constant__ CrossFrameLaunch L) {
-  __shared__ float part[8][33];
+constexpr int kEffWarps = 32;
+
+__global__ void __launch_bounds__(kEffWarps * 32) e_ff_kernel(const __grid_constant__ CrossFrameLaunch L) {
+  __shared__ float part[kEffWarps][33];
   __shared__ float give[32];
   const VideoInfo vi = L.videos[blockIdx.y];
   const int T = vi.n_vis / L.tokens_per_frame;
@@ -99,37 +123,36 @@ __global__ void __launch_bounds__(256) e_ff_kernel(const __grid_constant__ Cross
   const int t = t0 + lane;
   // Received: column t over the rows of frames a > t (row index a - 1 >= t).
   float recv = 0.f;
-  for (int ra = t0 + warp; ra <= T - 2; ra += 8)
-    if (t <= T - 2 && ra >= t) recv += A[static_cast<int64_t>(ra) * (T - 1) + t];
+  if (t <= T - 2) {
+#pragma unroll 4
+    for (int ra = t0 + warp; ra <= T - 2; ra += kEffWarps)
+      if (ra >= t) recv += A[static_cast<int64_t>(ra) * (T - 1) + t];
+  }
   part[warp][lane] = recv;
-  // Given: row t - 1 over the frames b < t.
-  for (int tt = warp; tt < 32; tt += 8) {
-    const int tg = t0 + tt;
+  // Given: row t - 1 over the frames b < t, one warp per frame.
+  {
+    const int tg = t0 + warp;
     float g = 0.f;
-    if (tg >= 1 && tg < T)
+    if (tg >= 1 && tg < T) {
+#pragma unroll 4
       for (int b = lane; b < tg; b += 32) g += A[static_cast<int64_t>(tg - 1) * (T - 1) + b];
+    }
     for (int off = 16; off > 0; off >>= 1) g += __shfl_xor_sync(kFull, g, off);
-    if (lane == 0) give[tt] = g;
+    if (lane == 0) give[warp] = g;
   }
   __syncthreads();
   if (warp == 0 && t < T) {
     float r = 0.f;
 #pragma unroll
-    for (int w = 0; w < 8; ++w) r += part[w][lane];
+    for (int w = 0; w < kEffWarps; ++w) r += part[w][lane];
     L.eff[vi.frame_off + t] = 0.5f * (give[lane] + r);
   }
 }
 
 template <int TILE>
 cudaError_t launch_pairs(const CrossFrameLaunch& L, cudaStream_t stream) {
-  const size_t smem = static_cast<size_t>(L.hq) * TILE * sizeof(float);
-  auto kern = cross_frame_pairs_kernel<TILE>;
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-  }
-  dim3 grid(L.n_rows, (L.max_kv + kKvPerCta - 1) / kKvPerCta);
-  kern<<<grid, TILE, smem, stream>>>(L);
+  dim3 grid(L.n_rows, (L.max_kv * L.fpt + kUnits - 1) / kUnits);
+  cross_frame_pairs_kernel<TILE><<<grid, TILE, 0, stream>>>(L);
   return cudaGetLastError();
 }
 
@@ -144,7 +167,7 @@ cudaError_t launch_cross_frame(const CrossFrameLaunch& L, cudaStream_t stream) {
   }
   if (L.eff && L.n_videos > 0 && L.max_frames > 0) {
     dim3 grid((L.max_frames + 31) / 32, L.n_videos);
-    e_ff_kernel<<<grid, 256, 0, stream>>>(L);
+    e_ff_kernel<<<grid, kEffWarps * 32, 0, stream>>>(L);
     return cudaGetLastError();
   }
   return cudaSuccess;
