@@ -396,6 +396,33 @@ def bench_ours(args, cfg):
     if status != 0:
         raise RuntimeError("device status reported an error")
 
+    # The step with the recompute evidence pass (text_evidence = 1): the probe
+    # without the text-row logit spill, then the evidence formed from Q, K and
+    # the LSE on the tensor cores. Same outputs; timed like the step.
+    ws_te = ev.Workspace()
+    maps_te = [torch.zeros_like(m) for m in maps]
+    ev.evisel_probe_attention(*pargs, ws=ws_te, o=o_cf, lse=lse_cf, text_evidence=True)
+
+    def probe_te():
+        ev.evisel_probe_attention(*pargs, ws=ws_te, o=o_cf, lse=lse_cf, text_evidence=True)
+
+    def evid_te():
+        ev.evisel_evidence_reduce(ws_te, hq, probe.n_vis, npf, len(probe.n_vis), tok=maps_te[0],
+                                  frame=maps_te[1], head=maps_te[2], aqf=maps_te[3])
+
+    def step_te():
+        probe_te()
+        evid_te()
+
+    te_step_ms = _time(step_te)
+    te_probe_ms = _time(probe_te)
+    te_ev_ms = _time(evid_te)
+    status = ev.evisel_status(ws_te)
+    te_ws_bytes = ws_te.nbytes
+    ws_te.free()
+    if status != 0:
+        raise RuntimeError("device status reported an error")
+
     line = None
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
@@ -416,6 +443,9 @@ def bench_ours(args, cfg):
                 "intra_frame": {"ms": if_ms, "gbs": if_bytes / (if_ms * 1e-3) / 1e9,
                                 "frac_of_hbm": if_bytes / (if_ms * 1e-3) / 1e9 / peaks["hbm"], "bytes": if_bytes,
                                 "tflops": if_flop / (if_ms * 1e-3) / 1e12},
+                "text_evidence_recompute": {"step_ms": te_step_ms, "probe_ms": te_probe_ms, "evidence_ms": te_ev_ms,
+                                            "tflops": st["flop"] / (te_step_ms * 1e-3) / 1e12,
+                                            "workspace_bytes": te_ws_bytes},
                 "cross_frame": {"probe_ms": pcf_ms, "probe_partials_bytes": fspill_bytes,
                                 "probe_overhead_ms": pcf_ms - attn_avg,
                                 "ms": cf_ms, "gbs": cf_bytes / (cf_ms * 1e-3) / 1e9,

@@ -95,6 +95,13 @@ typedef struct {
                                     hq * nnz(mask) * tile * (tile / min(N_v, 64))
                                     * 4 bytes).
                                     0: not kept. Ignored by evisel_intra_frame_evidence. */
+  int32_t text_evidence;         /* how evisel_evidence_reduce() forms the text-row
+                                    probabilities: 0 = from the text rows' logits the
+                                    probe spills into the workspace (hq * n_text *
+                                    n_vis * 4 bytes per video); 1 = recomputed from
+                                    q and k (no spill; q and k, like lse, must stay
+                                    alive until evisel_evidence_reduce() ran). Same
+                                    outputs within fp32 rounding. */
 } evisel_probe_args;
 
 /* Block-sparse causal GQA varlen attention (Eq. 1; Appendix Eq. 8 and Eq. 11

@@ -45,6 +45,7 @@ class ProbeArgs(ctypes.Structure):
         ("o", ctypes.c_void_p),
         ("lse", ctypes.c_void_p),
         ("cross_frame", ctypes.c_int32),
+        ("text_evidence", ctypes.c_int32),
     ]
 
 
@@ -129,7 +130,7 @@ class Workspace:
 
 
 def make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
-              softmax_scale=0.0, cross_frame=False):
+              softmax_scale=0.0, cross_frame=False, text_evidence=False):
     """Fills the C struct; returns (struct, keepalive) - keepalive holds the host arrays."""
     cu, cu_p = _i32(cu_seqlens)
     nv, nv_p = _i32(n_vis)
@@ -150,13 +151,17 @@ def make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_i
     a.mask_col_idx_h = ci_p
     a.o, a.lse = o.data_ptr(), lse.data_ptr()
     a.cross_frame = int(bool(cross_frame))
+    a.text_evidence = int(bool(text_evidence))
     return a, (cu, nv, rp, ci)
 
 
 def evisel_probe_attention(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx,
-                           ws=None, o=None, lse=None, softmax_scale=0.0, stream=None, cross_frame=False):
+                           ws=None, o=None, lse=None, softmax_scale=0.0, stream=None, cross_frame=False,
+                           text_evidence=False):
     """Block-sparse GQA varlen probe attention. q/k/v: CUDA bf16 [N, H, d].
-    ``cross_frame`` also keeps the partials evisel_cross_frame_evidence reads.
+    ``cross_frame`` also keeps the partials evisel_cross_frame_evidence reads;
+    ``text_evidence`` makes evisel_evidence_reduce recompute the text-row
+    probabilities from q and k instead of spilling the logits.
 
     Returns (o [N, hq, d] bf16, lse [hq, N] fp32, ws).
     """
@@ -173,7 +178,7 @@ def evisel_probe_attention(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, r
     if ws is None:
         ws = Workspace()
     args, keep = make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
-                           softmax_scale, cross_frame)
+                           softmax_scale, cross_frame, text_evidence)
     _check(lib.evisel_probe_attention(ctypes.byref(args), _stream_handle(stream), ctypes.byref(ws.ptr)))
     del keep
     return o, lse, ws
@@ -216,18 +221,19 @@ NOALLOC_SCRATCH_BYTES = 64 << 20
 
 def evisel_probe_evidence_noalloc(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
                                   tok, frame, head, aqf, accumulate=False, softmax_scale=0.0, stream=None,
-                                  wait_status=True):
+                                  wait_status=True, text_evidence=False):
     """Probe + evidence through the entry point that allocates nothing.
 
     For callers that cannot let the library call cudaMalloc: every output
     (o, lse and the four maps) is passed in, and the library's scratch is a
-    fixed 64 MiB static device array (problems that need more are rejected).
+    fixed 64 MiB static device array (problems that need more are rejected;
+    ``text_evidence`` drops the text-row logit spill, the largest part).
     Returns the device status word when ``wait_status`` (the call then waits
     for the stream), else None.
     """
     lib = load()
     args, keep = make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
-                           softmax_scale)
+                           softmax_scale, text_evidence=text_evidence)
     status = ctypes.c_int(0)
     _check(lib.evisel_probe_evidence_noalloc(ctypes.byref(args), tok.data_ptr(), frame.data_ptr(), head.data_ptr(),
                                              aqf.data_ptr(), int(bool(accumulate)), _stream_handle(stream),

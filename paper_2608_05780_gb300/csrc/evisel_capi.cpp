@@ -74,6 +74,7 @@ struct Plan {
   int total_vis = 0;
   int total_frames = 0;
   int n_tok = 0;
+  bool text_recompute = false;      // args->text_evidence: no spill, evidence from q and k
   // cross-frame partials (args->cross_frame)
   bool cross_frame = false;
   std::vector<VisRow> vrows;        // visual row tiles in mask order
@@ -102,6 +103,7 @@ int validate(const evisel_probe_args* a) {
   if (!(a->softmax_scale >= 0.f) || !std::isfinite(a->softmax_scale))
     return fail(EVISEL_EINVAL, "softmax_scale must be finite and >= 0");
   if (a->cross_frame != 0 && a->cross_frame != 1) return fail(EVISEL_EINVAL, "cross_frame must be 0 or 1");
+  if (a->text_evidence != 0 && a->text_evidence != 1) return fail(EVISEL_EINVAL, "text_evidence must be 0 or 1");
   if (a->cross_frame && npf < 16)
     return fail(EVISEL_EUNSUPPORTED, "cross-frame partials need tokens_per_frame >= 16");
   if (a->num_videos == 0) return EVISEL_OK;
@@ -173,12 +175,13 @@ void build_plan(const evisel_probe_args* a, Plan& P) {
     v.spill_off = spill;
     v.vis_off = vis_off;
     v.frame_off = frame_off;
-    spill += static_cast<int64_t>(hq) * v.n_vis * v.text_pitch;
+    if (!a->text_evidence) spill += static_cast<int64_t>(hq) * v.n_vis * v.text_pitch;
     vis_off += v.n_vis;
     frame_off += v.n_vis / a->tokens_per_frame;
     P.videos.push_back(v);
   }
   P.spill_floats = spill;
+  P.text_recompute = a->text_evidence != 0;
   P.total_vis = vis_off;
   P.total_frames = frame_off;
 
@@ -357,6 +360,10 @@ struct evisel_ws {
   // last probe, for the evidence pass
   bool probed = false;
   const float* lse = nullptr;
+  const void* q = nullptr;          // the probe's q and k (read by the recompute evidence)
+  const void* k = nullptr;
+  int hkv = 0, head_dim = 0;
+  float scale = 0.f;
   int hq = 0;
   int tokens_per_frame = 0;
   cudaStream_t last_stream = nullptr;
@@ -365,7 +372,8 @@ struct evisel_ws {
 namespace {
 
 std::vector<int32_t> plan_key(const evisel_probe_args* a) {
-  std::vector<int32_t> k = {a->num_videos, a->tokens_per_frame, a->hq, a->hkv, a->head_dim, a->tile, a->cross_frame};
+  std::vector<int32_t> k = {a->num_videos, a->tokens_per_frame, a->hq, a->hkv, a->head_dim, a->tile, a->cross_frame,
+                            a->text_evidence};
   for (int b = 0; b <= a->num_videos && a->num_videos > 0; ++b) k.push_back(a->cu_seqlens_h[b]);
   for (int b = 0; b < a->num_videos; ++b) k.push_back(a->n_vis_h[b]);
   int64_t rows = 0;
@@ -525,7 +533,7 @@ int evisel_probe_attention(const evisel_probe_args* args, void* stream_ptr, evis
     L.videos = ws->d_videos;
     L.o = args->o;
     L.lse = args->lse;
-    L.spill = ws->d_spill;
+    L.spill = P.text_recompute ? nullptr : ws->d_spill;
     L.part_o = ws->d_part_o;
     L.part_ml = ws->d_part_ml;
     L.status = ws->status;
@@ -563,6 +571,11 @@ int evisel_probe_attention(const evisel_probe_args* args, void* stream_ptr, evis
   }
   ws->probed = true;
   ws->lse = args->lse;
+  ws->q = args->q;
+  ws->k = args->k;
+  ws->hkv = args->hkv;
+  ws->head_dim = args->head_dim;
+  ws->scale = scale;
   ws->hq = args->hq;
   ws->tokens_per_frame = args->tokens_per_frame;
   ws->last_stream = stream;
@@ -598,6 +611,34 @@ int evisel_evidence_reduce(const evisel_ws* ws_c, float* tok, float* frame, floa
   L.total_vis = P.total_vis;
   L.total_frames = P.total_frames;
   L.accumulate = accumulate != 0;
+  if (P.text_recompute) {
+    // Token and frame maps from q and k (no spill); the finalize below forms
+    // the head map and A_qf from the frame map.
+    TextEvidenceLaunch T;
+    std::memset(&T, 0, sizeof(T));
+    int rc = encode_map(&T.tm_q, ws->q, P.n_tok, ws->hq, ws->head_dim, 128);
+    if (rc == EVISEL_OK) rc = encode_map(&T.tm_k, ws->k, P.n_tok, ws->hkv, ws->head_dim, 128);
+    if (rc != EVISEL_OK) return rc;
+    T.chunks = ws->d_chunks;
+    T.videos = ws->d_videos;
+    T.lse = ws->lse;
+    T.tok = tok;
+    T.frame = frame;
+    T.status = ws->status;
+    T.n_chunks = static_cast<int>(P.chunks.size());
+    T.n_tok = P.n_tok;
+    T.hq = ws->hq;
+    T.hkv = ws->hkv;
+    T.head_dim = ws->head_dim;
+    T.tokens_per_frame = ws->tokens_per_frame;
+    T.total_vis = P.total_vis;
+    T.total_frames = P.total_frames;
+    T.scale_log2 = ws->scale * 1.4426950408889634f;
+    T.accumulate = accumulate != 0;
+    cudaError_t te = launch_text_evidence(T, stream);
+    if (te != cudaSuccess) return cuda_fail(te, "text_evidence launch");
+    L.n_chunks = 0;
+  }
   cudaError_t e = launch_evidence(L, stream);
   if (e != cudaSuccess) return cuda_fail(e, "evidence launch");
   ws->last_stream = stream;

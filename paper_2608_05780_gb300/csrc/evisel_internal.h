@@ -166,7 +166,23 @@ struct CrossFrameLaunch {
   int accumulate;
 };
 
+// Text-row evidence by recompute (no logit spill): one CTA per (128 visual
+// keys, KV group).
+struct TextEvidenceLaunch {
+  CUtensorMap tm_q, tm_k;           // 3-D maps {d, heads, tokens}, box {64, 1, 128}, 128B swizzle
+  const EvChunk* chunks;
+  const VideoInfo* videos;
+  const float* lse;                 // [hq, N]
+  float* tok;                       // [hq, total_vis]
+  float* frame;                     // [hq, total_frames]
+  int* status;
+  int n_chunks, n_tok, hq, hkv, head_dim, tokens_per_frame, total_vis, total_frames;
+  float scale_log2;
+  int accumulate;
+};
+
 cudaError_t launch_intra_frame(const IntraFrameLaunch& L, cudaStream_t stream);
+cudaError_t launch_text_evidence(const TextEvidenceLaunch& L, cudaStream_t stream);
 cudaError_t launch_cross_frame(const CrossFrameLaunch& L, cudaStream_t stream);
 cudaError_t launch_probe_attn(const ProbeLaunch& L, cudaStream_t stream);
 cudaError_t launch_attn_combine(const CombineLaunch& L, cudaStream_t stream);

@@ -87,7 +87,7 @@ void make_plan(const evisel_probe_args* a, Counts& c, const Out* o) {
     v.spill_off = spill;
     v.vis_off = vis_off;
     v.frame_off = frame_off;
-    spill += static_cast<int64_t>(hq) * v.n_vis * v.text_pitch;
+    if (!a->text_evidence) spill += static_cast<int64_t>(hq) * v.n_vis * v.text_pitch;
     vis_off += v.n_vis;
     frame_off += v.n_vis / a->tokens_per_frame;
     if (o) o->videos[b] = v;
@@ -257,7 +257,7 @@ extern "C" int evisel_probe_evidence_noalloc(const evisel_probe_args* args, floa
     L.videos = reinterpret_cast<const VideoInfo*>(base + o_videos);
     L.o = args->o;
     L.lse = args->lse;
-    L.spill = reinterpret_cast<float*>(base + o_spill);
+    L.spill = args->text_evidence ? nullptr : reinterpret_cast<float*>(base + o_spill);
     L.part_o = reinterpret_cast<float*>(base + o_part_o);
     L.part_ml = reinterpret_cast<float2*>(base + o_part_ml);
     L.status = reinterpret_cast<int*>(base);
@@ -308,6 +308,37 @@ extern "C" int evisel_probe_evidence_noalloc(const evisel_probe_args* args, floa
     E.total_vis = c.total_vis;
     E.total_frames = c.total_frames;
     E.accumulate = accumulate != 0;
+    if (args->text_evidence && c.chunks > 0) {
+      // Token and frame maps recomputed from q and k (no spill).
+      TextEvidenceLaunch T;
+      std::memset(&T, 0, sizeof(T));
+      rc = encode_tensor_map(&T.tm_q, args->q, n_tok, args->hq, args->head_dim, 128);
+      if (rc == EVISEL_OK) rc = encode_tensor_map(&T.tm_k, args->k, n_tok, args->hkv, args->head_dim, 128);
+      if (rc != EVISEL_OK) return rc;
+      T.chunks = E.chunks;
+      T.videos = E.videos;
+      T.lse = args->lse;
+      T.tok = tok;
+      T.frame = frame;
+      T.status = reinterpret_cast<int*>(base);
+      T.n_chunks = static_cast<int>(c.chunks);
+      T.n_tok = n_tok;
+      T.hq = args->hq;
+      T.hkv = args->hkv;
+      T.head_dim = args->head_dim;
+      T.tokens_per_frame = args->tokens_per_frame;
+      T.total_vis = c.total_vis;
+      T.total_frames = c.total_frames;
+      const float scale = args->softmax_scale > 0.f ? args->softmax_scale : 1.0f / std::sqrt(float(args->head_dim));
+      T.scale_log2 = scale * 1.4426950408889634f;
+      T.accumulate = accumulate != 0;
+      e = launch_text_evidence(T, stream);
+      if (e != cudaSuccess) {
+        cudaGetLastError();
+        return set_last_error(EVISEL_ECUDA, (std::string("text_evidence launch: ") + cudaGetErrorString(e)).c_str());
+      }
+      E.n_chunks = 0;
+    }
     e = launch_evidence(E, stream);
     if (e != cudaSuccess) {
       cudaGetLastError();

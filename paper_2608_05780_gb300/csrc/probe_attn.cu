@@ -363,7 +363,7 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
   const int qpos = it.q_start + row_local;
   const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
   const uint32_t tmem = tmem_base + lane_base + slot * C::SLOT_COLS;
-  const bool spill_rows = it.text_row0 >= 0 && row_ok;
+  const bool spill_rows = it.text_row0 >= 0 && row_ok && L.spill != nullptr;   // no spill: evidence recomputed
   // With one slot, S alternates between both slots' S columns (see the MMA issuer).
   const bool two = left > C::HP;
 

@@ -27,13 +27,15 @@ def to_device(probe):
     return q, k, v
 
 
-def run_cuda(ev, probe, ws=None, maps=None, accumulate=False, qkv=None):
-    """Probe + evidence on the GPU; returns numpy outputs and the workspace."""
+def run_cuda(ev, probe, ws=None, maps=None, accumulate=False, qkv=None, text_evidence=False):
+    """Probe + evidence on the GPU; returns numpy outputs and the workspace.
+    ``text_evidence``: the evidence recomputed from q and k instead of the spill."""
     import torch
     cfg = probe.cfg
     q, k, v = qkv if qkv is not None else to_device(probe)
     o, lse, ws = ev.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame,
-                                           cfg.tile, probe.row_ptr, probe.col_idx, ws=ws)
+                                           cfg.tile, probe.row_ptr, probe.col_idx, ws=ws,
+                                           text_evidence=text_evidence)
     kw = {}
     if maps is not None:
         kw = dict(tok=maps[0], frame=maps[1], head=maps[2], aqf=maps[3])
