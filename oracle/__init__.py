@@ -13,10 +13,15 @@ Every function here follows the paper's statement of the probe:
   * logits q k^T / sqrt(d) (Eq. 8) and row-wise normalisation (Eq. 11);
   * head averaging, the query-frame cue A_qf, the intra-frame cue A_if and
     the cross-frame cue A_ff with its timestamp-aligned E_ff (Sec. 3.2,
-    "Evidence Decomposition").
+    "Evidence Decomposition");
+  * the top-p block retention of the sparse prefill (Appendix, Eq. 6-9) and
+    attention restricted to the retained blocks (``topp``).
 Parity pins for each function live in ``tests/test_oracle_pins.py``.
 """
 from .attention import (  # noqa: F401
     token_layout, allowed_row, probe_rows, probe, text_probabilities, evidence, intra_frame, frame_mass_rows,
     cross_frame, e_ff,
+)
+from .topp import (  # noqa: F401
+    block_layout, block_means, select_prefix, retained_blocks, attended_mask, probe_rows_topp,
 )

@@ -13,6 +13,7 @@ Each test names the pin it realises:
   O9  planted frames rank top on the head-summed frame map
   O10 linearity of O in V
   F1-F4 the intra-frame cue A_if (closed form, dense weights, brute force, structure)
+  H1-H5 top-p block retention (closed form, brute force, planted block, limits, keep-all)
   G1-G5 the cross-frame cue A_ff and E_ff (closed form, mass balance with A_if, brute force,
         dense weights, a hand-worked E_ff)
 """
@@ -587,3 +588,135 @@ def test_G1_catches_a_block_mean_over_all_pairs(monkeypatch):
     monkeypatch.setattr(op, "frame_mass_rows", per_entry)
     with pytest.raises(AssertionError):
         test_G1_cross_frame_constant_keys()
+
+
+# ---------------------------------------------------------------- top-p block retention (Eq. 6-9)
+# Pins of oracle.topp:
+#   H1  constant keys: uniform p over H_i, so S_i is the ceil(tau |H_i|)
+#       lowest block ids (the tie rule), counted without any softmax
+#   H2  brute force, pure-Python block means, logits, softmax and sort
+#   H3  a planted block aligned with the row's query takes all the mass
+#   H4  monotone in tau; tau -> 1 keeps all of H_i; tiny tau keeps the argmax
+#   H5  keeping every block equals dense causal attention (torch, float64)
+def _topp_case(seed, videos=((32, 9), (24, 5)), hq=4, hkv=2, d=8, block=4):
+    rng = np.random.default_rng(seed)
+    n_vis = np.array([a for a, _ in videos], np.int32)
+    lens = np.array([a + b for a, b in videos])
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    n = int(cu[-1])
+    q = wl.bf16_round(rng.standard_normal((n, hq, d)).astype(np.float32))
+    k = wl.bf16_round(rng.standard_normal((n, hkv, d)).astype(np.float32))
+    v = wl.bf16_round(rng.standard_normal((n, hkv, d)).astype(np.float32))
+    return dict(q=q, k=k, v=v, cu=cu, n_vis=n_vis, block=block)
+
+
+def test_H1_topp_constant_keys():
+    c = _topp_case(41)
+    k = np.broadcast_to(c["k"][0:1], c["k"].shape).copy()
+    tau = 0.93          # tau * n stays away from integers for n <= 15 (no cumulative-sum rounding ties)
+    sets, probs = oracle.retained_blocks(c["q"], k, c["cu"], c["n_vis"], 4, tau)
+    for b in range(2):
+        s0, s1, nv = int(c["cu"][b]), int(c["cu"][b + 1]), int(c["n_vis"][b])
+        nb = nv // 4 + -(-(s1 - s0 - nv) // 4)
+        for row in range(s0, s1):
+            # blocks ending before the row: every block whose start + length <= local position
+            n_hist = sum(1 for s, ln in oracle.block_layout(nv, s1 - s0 - nv, 4) if s + ln <= row - s0)
+            assert n_hist <= nb
+            want = list(range(math.ceil(tau * n_hist))) if n_hist else []
+            for h in range(4):
+                assert sets[(h, row)] == want, (b, row, h)
+
+
+@pytest.mark.parametrize("seed", [42, 43])
+def test_H2_topp_brute_force(seed):
+    c = _topp_case(seed, videos=((16, 7), (12, 3)), d=5, block=4)
+    tau = 0.8
+    sets, _ = oracle.retained_blocks(c["q"], c["k"], c["cu"], c["n_vis"], 4, tau)
+    q, k = c["q"], c["k"]
+    hq, hkv = q.shape[1], k.shape[1]
+    for b in range(2):
+        s0, s1, nv = int(c["cu"][b]), int(c["cu"][b + 1]), int(c["n_vis"][b])
+        blocks = [(s, 4) for s in range(0, nv, 4)] + [(nv + s, min(4, s1 - s0 - nv - s)) for s in range(0, s1 - s0 - nv, 4)]
+        for row in range(s0, s1):
+            for h in range(hq):
+                g = []
+                for j, (s, ln) in enumerate(blocks):
+                    if s + ln > row - s0:
+                        continue
+                    kb = [sum(float(k[s0 + s + t, h * hkv // hq, e]) for t in range(ln)) / ln for e in range(5)]
+                    g.append((j, sum(float(q[row, h, e]) * kb[e] for e in range(5)) / math.sqrt(5)))
+                if not g:
+                    assert sets[(h, row)] == []
+                    continue
+                mx = max(x for _, x in g)
+                z = sum(math.exp(x - mx) for _, x in g)
+                ranked = sorted(((-math.exp(x - mx) / z, j) for j, x in g))
+                acc, keep = 0.0, []
+                for negp, j in ranked:
+                    if acc >= tau:
+                        break
+                    keep.append(j)
+                    acc += -negp
+                assert sets[(h, row)] == sorted(keep), (b, row, h)
+
+
+def test_H3_topp_planted_block_takes_the_mass():
+    c = _topp_case(44, videos=((32, 6),), hq=2, hkv=2)
+    q, k = c["q"], c["k"].copy()
+    row = 35                                          # a text row; block 3 (tokens 12..15) is planted
+    for h in range(2):
+        k[12:16, h, :] = 40.0 * q[row, h, :] / np.linalg.norm(q[row, h, :])
+    sets, probs = oracle.retained_blocks(q, k, c["cu"], c["n_vis"], 4, 0.97, rows=[row])
+    for h in range(2):
+        assert sets[(h, row)] == [3], h
+
+
+def test_H4_topp_monotone_and_limits():
+    c = _topp_case(45)
+    args = (c["q"], c["k"], c["cu"], c["n_vis"], 4)
+    rows = [10, 20, 33, 40, 55, 60]
+    s_lo, _ = oracle.retained_blocks(*args, 0.5, rows=rows)
+    s_hi, probs = oracle.retained_blocks(*args, 0.95, rows=rows)
+    s_all, _ = oracle.retained_blocks(*args, 1.0 - 1e-12, rows=rows)
+    s_one, _ = oracle.retained_blocks(*args, 1e-9, rows=rows)
+    for key in s_lo:
+        hist, p = probs[key]
+        assert set(s_lo[key]) <= set(s_hi[key]) <= set(s_all[key])
+        assert s_all[key] == [int(j) for j in hist]
+        assert s_one[key] == ([int(hist[np.argmax(p)])] if hist.size else [])
+        if hist.size:
+            kept = np.isin(hist, s_hi[key])
+            assert p[kept].sum() >= 0.95 - 1e-12
+            assert p[kept].sum() - p[kept].min() < 0.95            # minimal
+            assert p[kept].min() >= p[~kept].max(initial=0.0)       # a top set
+
+
+def test_H5_topp_keep_all_equals_dense_causal():
+    torch = pytest.importorskip("torch")
+    c = _topp_case(46, videos=((16, 5),))
+    rows = np.arange(21)
+    sets, probs = oracle.retained_blocks(c["q"], c["k"], c["cu"], c["n_vis"], 4, 1.0 - 1e-12, rows=rows)
+    o, lse = oracle.probe_rows_topp(c["q"], c["k"], c["v"], c["cu"], c["n_vis"], 4, sets, rows)
+    qt = torch.from_numpy(c["q"].astype(np.float64)).transpose(0, 1)
+    kt = torch.from_numpy(c["k"].astype(np.float64)).transpose(0, 1).repeat_interleave(2, 0)
+    vt = torch.from_numpy(c["v"].astype(np.float64)).transpose(0, 1).repeat_interleave(2, 0)
+    ref = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True).transpose(0, 1).numpy()
+    np.testing.assert_allclose(o, ref, atol=1e-12)
+
+
+def test_H3_catches_an_ascending_order(monkeypatch):
+    """Planted mistake: ranking H_i by p ascending."""
+    import oracle.topp as ot
+
+    def ascending(p, tau):
+        order = sorted(range(len(p)), key=lambda j: (p[j], j))
+        acc, keep = 0.0, []
+        for j in order:
+            if acc >= tau:
+                break
+            keep.append(j)
+            acc += p[j]
+        return sorted(keep)
+    monkeypatch.setattr(ot, "select_prefix", ascending)
+    with pytest.raises(AssertionError):
+        test_H3_topp_planted_block_takes_the_mass()
