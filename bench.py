@@ -451,6 +451,28 @@ def bench_ours(args, cfg):
         evid_te()
 
     te_step_ms = _time(step_te)
+
+    # The top-p block retention of the sparse prefill (Appendix Eq. 6-9) on the
+    # same inputs, blocks of N_v tokens, tau_p = 0.97 (outside the step: the
+    # workloads' masks are static).
+    ws_tp = ev.Workspace()
+    keep_tp, uni_tp, ws_tp = ev.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, npf, 0.97,
+                                                 ws=ws_tp)
+
+    def topp():
+        ev.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, npf, 0.97, ws=ws_tp)
+
+    tp_ms = _time(topp)
+    status = ev.evisel_status(ws_tp)
+    ws_tp.free()
+    del keep_tp, uni_tp
+    if status != 0:
+        raise RuntimeError("device status reported an error")
+    n_blk = int(sum(int(nv) // npf + -(-int(nt) // npf) for nv, nt in zip(probe.n_vis, probe.n_text)))
+    # algorithmic tensor work: 4 passes of q k_bar^T over each row's history, head by head
+    tp_flop = 4 * 2.0 * d * hq * sum(
+        sum((p_ // npf) for p_ in range(int(nv))) + sum(int(nv) // npf + t // npf for t in range(int(nt)))
+        for nv, nt in zip(probe.n_vis, probe.n_text))
     te_probe_ms = _time(probe_te)
     te_ev_ms = _time(evid_te)
     status = ev.evisel_status(ws_te)
@@ -479,6 +501,8 @@ def bench_ours(args, cfg):
                 "intra_frame": {"ms": if_ms, "gbs": if_bytes / (if_ms * 1e-3) / 1e9,
                                 "frac_of_hbm": if_bytes / (if_ms * 1e-3) / 1e9 / peaks["hbm"], "bytes": if_bytes,
                                 "tflops": if_flop / (if_ms * 1e-3) / 1e12},
+                "topp_mask": {"ms": tp_ms, "block": npf, "tau_p": 0.97, "blocks": n_blk,
+                              "tflops_history": tp_flop / (tp_ms * 1e-3) / 1e12},
                 "text_evidence_recompute": {"step_ms": te_step_ms, "probe_ms": te_probe_ms, "evidence_ms": te_ev_ms,
                                             "tflops": st["flop"] / (te_step_ms * 1e-3) / 1e12,
                                             "workspace_bytes": te_ws_bytes},

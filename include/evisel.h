@@ -239,6 +239,37 @@ int evisel_cross_frame_evidence(const evisel_probe_args* args, evisel_ws* ws, fl
                                 int accumulate, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * evisel_topp_mask: the top-p block retention of the sparse prefill (Appendix,
+ * "Detailed Sparse Prefilling", Eq. 6-9 and the retention rule after Eq. 9).
+ * Blocks: per video, visual blocks of `block` tokens from the visual start,
+ * then the text tokens in blocks of `block` from the text start (the last may
+ * be short); block ids count the visual blocks first. For row i: H_i = the
+ * blocks of its video that end before i; k_bar_j = mean key of block j (Eq. 7,
+ * per KV head, rounded to bf16); g_ij = softmax_scale q_i k_bar_j (Eq. 8);
+ * p_ij = softmax over H_i (Eq. 9); S_i = the shortest prefix of H_i ordered by
+ * p descending (ties: lower block id) whose mass reaches tau_p. Logits closer
+ * than (max - min) / 16384 over H_i may be taken as ties.
+ *   args   q, k, cu_seqlens_h, n_vis_h, tokens_per_frame, hq, hkv, head_dim,
+ *          tile, softmax_scale as for the probe (the mask, v, o, lse are not read).
+ *   block  B: a power of two, 16 <= B <= tokens_per_frame (so B divides N_v).
+ *   tau_p  in (0, 1] (the paper uses 0.97).
+ *   keep   device uint32 [hq, W, N_tot], W = ceil(max_b blocks_b / 32): bit j of
+ *          word w of (h, row) is block 32 w + j of the row's video, set for S_i
+ *          and for the row's own block (whose causal prefix it attends).
+ *   tile_union  device uint32 [R, ceil(max_b ceil(n_vis_b / tile) / 32)] or NULL:
+ *          for each visual row tile of the probe's tiling (R as the mask's rows),
+ *          bit c of the video-local visual kv tile c, set when some row of the
+ *          tile keeps a block of that tile for some head. Read as a CSR (each row
+ *          lists its set bits ascending), it is a valid mask for
+ *          evisel_probe_attention() whose kept tiles cover every row's S_i.
+ *   ws_inout  a workspace (created when *ws_inout == NULL) that holds the
+ *          call's metadata and the k_bar scratch.
+ * Asynchronous on `stream`. Errors: EVISEL_EINVAL, EVISEL_EUNSUPPORTED,
+ * EVISEL_ENOMEM, EVISEL_ECUDA; device timeouts through evisel_status(). */
+int evisel_topp_mask(const evisel_probe_args* args, int32_t block, float tau_p, uint32_t* keep,
+                     uint32_t* tile_union, void* stream, evisel_ws** ws_inout);
+
+/* ---------------------------------------------------------------------------
  * evisel_selftest_wait: failure detection check (no counterpart in the paper).
  * Every wait in the library's kernels is bounded: it gives up after a time
  * limit, records EVISEL_ETIMEOUT in a device status word and lets the kernel

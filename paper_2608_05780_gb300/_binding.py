@@ -85,6 +85,8 @@ def load(path: str = LIB_PATH):
     lib.evisel_intra_frame_evidence.restype = i32
     lib.evisel_cross_frame_evidence.argtypes = [ctypes.POINTER(ProbeArgs), vp, vp, vp, i32, vp]
     lib.evisel_cross_frame_evidence.restype = i32
+    lib.evisel_topp_mask.argtypes = [ctypes.POINTER(ProbeArgs), i32, ctypes.c_float, vp, vp, vp, ctypes.POINTER(vp)]
+    lib.evisel_topp_mask.restype = i32
     lib.evisel_selftest_wait.argtypes = [i32, i32, vp, ctypes.POINTER(ctypes.c_int)]
     lib.evisel_selftest_wait.restype = i32
     _lib = lib
@@ -294,3 +296,52 @@ def evisel_cross_frame_evidence(q, k, v, cu_seqlens, n_vis, tokens_per_frame, ti
                                            _stream_handle(stream)))
     del keep
     return aff, eff
+
+
+def evisel_topp_mask(q, k, cu_seqlens, n_vis, tokens_per_frame, tile, block, tau_p, ws=None, softmax_scale=0.0,
+                     stream=None, union=True):
+    """Top-p block retention (Appendix Eq. 6-9): returns (keep, tile_union, ws)
+    with keep int32 [hq, W, N] (uint32 bit words), tile_union int32
+    [visual row tiles, TW] or None."""
+    import torch
+    lib = load()
+    nv = np.asarray(n_vis, dtype=np.int64)
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    n_text = np.diff(cu) - nv
+    nb = nv // int(block) + -(-n_text // int(block))
+    n, hq = int(q.shape[0]), int(q.shape[1])
+    n_words = max(1, -(-int(nb.max() if nb.size else 0) // 32))
+    keep = torch.empty((hq, n_words, n), dtype=torch.int32, device=q.device)
+    n_vt = -(-nv // int(tile))
+    uni = None
+    if union:
+        uni = torch.empty((int(n_vt.sum()), max(1, -(-int(n_vt.max() if n_vt.size else 0) // 32))),
+                          dtype=torch.int32, device=q.device)
+    if ws is None:
+        ws = Workspace()
+    dummy = torch.empty(0, device=q.device)
+    args, keepalive = make_args(q, k, k, cu_seqlens, n_vis, tokens_per_frame, tile, [0], [], dummy, dummy,
+                                softmax_scale)
+    _check(lib.evisel_topp_mask(ctypes.byref(args), int(block), float(tau_p), keep.data_ptr(),
+                                uni.data_ptr() if uni is not None and uni.numel() else None,
+                                _stream_handle(stream), ctypes.byref(ws.ptr)))
+    del keepalive
+    return keep, uni, ws
+
+
+def tile_union_to_csr(tile_union, n_vis, tile):
+    """Host CSR (row_ptr, col_idx) of a tile union from evisel_topp_mask."""
+    bits = tile_union.cpu().numpy().view(np.uint32)
+    row_ptr, cols = [0], []
+    r = 0
+    for nv in np.asarray(n_vis, dtype=np.int64):
+        for _ in range(-(-int(nv) // int(tile))):
+            for w, word in enumerate(bits[r]):
+                word = int(word)
+                while word:
+                    low = word & -word
+                    cols.append(w * 32 + low.bit_length() - 1)
+                    word ^= low
+            row_ptr.append(len(cols))
+            r += 1
+    return np.array(row_ptr, np.int32), np.array(cols, np.int32)

@@ -367,6 +367,12 @@ struct evisel_ws {
   int hq = 0;
   int tokens_per_frame = 0;
   cudaStream_t last_stream = nullptr;
+  // top-p mask builder: [videos | row tiles | k_bar] on the device, staged through pinned memory
+  void* topp_buf = nullptr;
+  size_t topp_bytes = 0;
+  void* topp_stage = nullptr;
+  size_t topp_stage_bytes = 0;
+  cudaEvent_t topp_done = nullptr;
 };
 
 namespace {
@@ -741,6 +747,143 @@ int evisel_cross_frame_evidence(const evisel_probe_args* args, evisel_ws* ws, fl
   return EVISEL_OK;
 }
 
+int evisel_topp_mask(const evisel_probe_args* a, int32_t block, float tau_p, uint32_t* keep, uint32_t* tile_union,
+                     void* stream_ptr, evisel_ws** ws_inout) {
+  g_last_error.clear();
+  if (!a) return fail(EVISEL_EINVAL, "args is NULL");
+  if (!ws_inout) return fail(EVISEL_EINVAL, "ws_inout is NULL");
+  if (a->num_videos < 0 || (a->num_videos > 0 && (!a->cu_seqlens_h || !a->n_vis_h)))
+    return fail(EVISEL_EINVAL, "num_videos / cu_seqlens_h / n_vis_h");
+  if (a->head_dim != 64 && a->head_dim != 128) return fail(EVISEL_EUNSUPPORTED, "head_dim must be 64 or 128");
+  if (a->tile != 64 && a->tile != 128) return fail(EVISEL_EUNSUPPORTED, "tile must be 64 or 128");
+  if (a->hq < 1 || a->hkv < 1 || a->hq % a->hkv != 0) return fail(EVISEL_EUNSUPPORTED, "hq must be a multiple of hkv");
+  const int npf = a->tokens_per_frame;
+  if (npf < 4 || npf > a->tile || (npf & (npf - 1)) != 0)
+    return fail(EVISEL_EUNSUPPORTED, "tokens_per_frame must be a power of two in [4, tile]");
+  if (block < 16 || block > npf || (block & (block - 1)) != 0)
+    return fail(EVISEL_EUNSUPPORTED, "block must be a power of two in [16, tokens_per_frame] (it divides N_v)");
+  if (!(tau_p > 0.f && tau_p <= 1.f)) return fail(EVISEL_EINVAL, "tau_p must be in (0, 1]");
+  if (!(a->softmax_scale >= 0.f) || !std::isfinite(a->softmax_scale))
+    return fail(EVISEL_EINVAL, "softmax_scale must be finite and >= 0");
+  if (a->num_videos == 0) return EVISEL_OK;
+  if (a->cu_seqlens_h[0] != 0) return fail(EVISEL_EINVAL, "cu_seqlens[0] must be 0");
+  for (int b = 0; b < a->num_videos; ++b) {
+    const int64_t len = static_cast<int64_t>(a->cu_seqlens_h[b + 1]) - a->cu_seqlens_h[b];
+    if (len < 0 || a->n_vis_h[b] < 0 || a->n_vis_h[b] > len || a->n_vis_h[b] % npf != 0)
+      return fail(EVISEL_EINVAL, "cu_seqlens / n_vis of video " + std::to_string(b));
+  }
+  const int n_tok = a->cu_seqlens_h[a->num_videos];
+  if (n_tok == 0) return EVISEL_OK;
+  if (!a->q || !a->k || !keep) return fail(EVISEL_EINVAL, "q, k or keep is NULL");
+  if ((reinterpret_cast<uintptr_t>(a->q) & 15u) || (reinterpret_cast<uintptr_t>(a->k) & 15u))
+    return fail(EVISEL_EINVAL, "q and k must be 16-byte aligned");
+
+  // Videos, their blocks and row tiles (128 rows: the visual rows, then the text rows).
+  std::vector<ToppVideo> vids;
+  std::vector<ToppRowTile> tiles;
+  int blk_off = 0, row_tile0 = 0, max_blocks = 0, max_vis_tiles = 0;
+  for (int b = 0; b < a->num_videos; ++b) {
+    ToppVideo v{};
+    v.start = a->cu_seqlens_h[b];
+    v.n_vis = a->n_vis_h[b];
+    v.n_text = a->cu_seqlens_h[b + 1] - v.start - v.n_vis;
+    v.blk_off = blk_off;
+    v.row_tile0 = row_tile0;
+    const int nb = v.n_vis / block + (v.n_text + block - 1) / block;
+    blk_off += nb;
+    max_blocks = std::max(max_blocks, nb);
+    const int n_vt = (v.n_vis + a->tile - 1) / a->tile;
+    row_tile0 += n_vt;
+    max_vis_tiles = std::max(max_vis_tiles, n_vt);
+    for (int s = 0; s < v.n_vis; s += 128)
+      tiles.push_back(ToppRowTile{b, v.start + s, std::min(128, v.n_vis - s), s, 0, 0, 0, 0});
+    for (int s = 0; s < v.n_text; s += 128)
+      tiles.push_back(ToppRowTile{b, v.start + v.n_vis + s, std::min(128, v.n_text - s), v.n_vis + s, 1, 0, 0, 0});
+    vids.push_back(v);
+  }
+  const int n_words = std::max(1, (max_blocks + 31) / 32);
+  const int n_tile_words = std::max(1, (max_vis_tiles + 31) / 32);
+
+  if (!*ws_inout) {
+    int rc = create_ws(ws_inout);
+    if (rc != EVISEL_OK) return rc;
+  }
+  evisel_ws* ws = *ws_inout;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
+  const size_t meta = align_up(vids.size() * sizeof(ToppVideo), 256) + align_up(tiles.size() * sizeof(ToppRowTile), 256);
+  const size_t kbar_bytes = static_cast<size_t>(blk_off) * a->hkv * a->head_dim * 2;
+  const size_t need = meta + kbar_bytes;
+  if (!ws->topp_done && cudaEventCreateWithFlags(&ws->topp_done, cudaEventDisableTiming) != cudaSuccess)
+    return cuda_fail(cudaGetLastError(), "event");
+  cudaEventSynchronize(ws->topp_done);             // the staging buffer may still feed the last upload
+  if (need > ws->topp_bytes) {
+    cudaStreamSynchronize(ws->last_stream);
+    cudaStreamSynchronize(stream);
+    if (ws->topp_buf) cudaFree(ws->topp_buf);
+    ws->topp_buf = nullptr;
+    ws->topp_bytes = 0;
+    if (cudaMalloc(&ws->topp_buf, need) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(EVISEL_ENOMEM, "top-p scratch of " + std::to_string(need) + " bytes");
+    }
+    ws->topp_bytes = need;
+  }
+  if (meta > ws->topp_stage_bytes) {
+    if (ws->topp_stage) cudaFreeHost(ws->topp_stage);
+    ws->topp_stage = nullptr;
+    ws->topp_stage_bytes = 0;
+    if (cudaMallocHost(&ws->topp_stage, meta) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(EVISEL_ENOMEM, "top-p staging");
+    }
+    ws->topp_stage_bytes = meta;
+  }
+  char* h = static_cast<char*>(ws->topp_stage);
+  const size_t o_tiles = align_up(vids.size() * sizeof(ToppVideo), 256);
+  std::memcpy(h, vids.data(), vids.size() * sizeof(ToppVideo));
+  std::memcpy(h + o_tiles, tiles.data(), tiles.size() * sizeof(ToppRowTile));
+  char* d = static_cast<char*>(ws->topp_buf);
+  cudaError_t e = cudaMemcpyAsync(d, h, meta, cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaEventRecord(ws->topp_done, stream);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(keep, 0, static_cast<size_t>(a->hq) * n_words * n_tok * sizeof(uint32_t), stream);
+  const int r_vis = row_tile0;
+  if (e == cudaSuccess && tile_union && r_vis > 0)
+    e = cudaMemsetAsync(tile_union, 0, static_cast<size_t>(r_vis) * n_tile_words * sizeof(uint32_t), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "top-p upload");
+
+  ToppLaunch L;
+  std::memset(&L, 0, sizeof(L));
+  int rc = encode_map(&L.tm_q, a->q, n_tok, a->hq, a->head_dim, 128);
+  if (rc == EVISEL_OK && blk_off > 0) rc = encode_map(&L.tm_kbar, d + meta, blk_off, a->hkv, a->head_dim, 128);
+  if (rc != EVISEL_OK) return rc;
+  const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / std::sqrt(float(a->head_dim));
+  L.k = a->k;
+  L.kbar = d + meta;
+  L.vids = reinterpret_cast<const ToppVideo*>(d);
+  L.tiles = reinterpret_cast<const ToppRowTile*>(d + o_tiles);
+  L.keep = keep;
+  L.tile_union = tile_union;
+  L.status = ws->status;
+  L.n_videos = a->num_videos;
+  L.n_tiles = static_cast<int>(tiles.size());
+  L.n_blocks_total = blk_off;
+  L.n_words = n_words;
+  L.n_tile_words = n_tile_words;
+  L.n_tok = n_tok;
+  L.hq = a->hq;
+  L.hkv = a->hkv;
+  L.head_dim = a->head_dim;
+  L.block = block;
+  L.tile = a->tile;
+  L.scale_log2 = scale * 1.4426950408889634f;
+  L.tau = tau_p;
+  e = launch_topp(L, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "top-p launch");
+  ws->last_stream = stream;
+  return EVISEL_OK;
+}
+
 void evisel_free(evisel_ws* ws) {
   if (!ws) return;
   int prev = -1;
@@ -752,6 +895,10 @@ void evisel_free(evisel_ws* ws) {
   if (ws->status) cudaFree(ws->status);
   if (ws->stage) cudaFreeHost(ws->stage);
   if (ws->stage_done) cudaEventDestroy(ws->stage_done);
+  if (ws->topp_done) cudaEventSynchronize(ws->topp_done);
+  if (ws->topp_buf) cudaFree(ws->topp_buf);
+  if (ws->topp_stage) cudaFreeHost(ws->topp_stage);
+  if (ws->topp_done) cudaEventDestroy(ws->topp_done);
   if (prev >= 0 && prev != ws->device) cudaSetDevice(prev);
   cudaGetLastError();
   delete ws;

@@ -181,8 +181,43 @@ struct TextEvidenceLaunch {
   int accumulate;
 };
 
+// Top-p block retention (mask builder).
+struct ToppVideo {
+  int32_t start;      // global index of the video's first token
+  int32_t n_vis, n_text;
+  int32_t blk_off;    // global index of its first block (k_bar rows)
+  int32_t row_tile0;  // global index of its first visual row tile of the attention's tiling
+  int32_t pad0, pad1, pad2;
+};
+static_assert(sizeof(ToppVideo) == 32, "ToppVideo is 32 bytes");
+
+struct ToppRowTile {  // 128 rows of one video (visual rows, or text rows)
+  int32_t video;
+  int32_t q_start;    // global index of the first row
+  int32_t q_len;
+  int32_t local0;     // video-local position of the first row
+  int32_t text;       // 1: text rows
+  int32_t pad0, pad1, pad2;
+};
+static_assert(sizeof(ToppRowTile) == 32, "ToppRowTile is 32 bytes");
+
+struct ToppLaunch {
+  CUtensorMap tm_q, tm_kbar;        // q {d, hq, N}; k_bar {d, hkv, blocks}; boxes {64, 1, 128}
+  const void* k;                    // bf16 [N, hkv, d]
+  void* kbar;                       // bf16 [blocks, hkv, d]
+  const ToppVideo* vids;
+  const ToppRowTile* tiles;
+  uint32_t* keep;                   // [hq, n_words, N]
+  uint32_t* tile_union;             // [visual row tiles, n_tile_words] or null
+  int* status;
+  int n_videos, n_tiles, n_blocks_total, n_words, n_tile_words;
+  int n_tok, hq, hkv, head_dim, block, tile;
+  float scale_log2, tau;
+};
+
 cudaError_t launch_intra_frame(const IntraFrameLaunch& L, cudaStream_t stream);
 cudaError_t launch_text_evidence(const TextEvidenceLaunch& L, cudaStream_t stream);
+cudaError_t launch_topp(const ToppLaunch& L, cudaStream_t stream);
 cudaError_t launch_cross_frame(const CrossFrameLaunch& L, cudaStream_t stream);
 cudaError_t launch_probe_attn(const ProbeLaunch& L, cudaStream_t stream);
 cudaError_t launch_attn_combine(const CombineLaunch& L, cudaStream_t stream);

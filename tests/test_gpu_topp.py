@@ -1,0 +1,145 @@
+"""GPU parity of the top-p block retention (evisel_topp_mask) against
+oracle.topp.retained_blocks, through the C ABI.
+
+Several sets can be "the" answer only at ties, so each GPU set is checked
+against the oracle's p (block means rounded to bf16 as the tensor-core path
+takes them): it holds the row's own block and blocks of H_i only; its mass
+reaches tau_p; it is minimal (without its least block the mass is below
+tau_p); and it is a top set (no dropped block has a larger p). Each check
+allows EPS of p: the GPU's logits are fp32 sums of bf16 products, and its
+order resolves logits to (max - min) / 16384 over H_i.
+The tile union is checked bit for bit against the union of the GPU's own
+sets, and, read as a mask, it drives the probe, whose rows match the oracle.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_05780_gb300 import _binding as B
+from paper_2608_05780_gb300 import workloads as wl
+from gpu_helpers import check_lse, check_o, to_device
+
+pytestmark = pytest.mark.gpu
+
+EPS = 2e-5
+LOG2_EPS = 3e-5      # fp32 logits (bf16 products) against the oracle's float64, in log2 units
+
+
+def _gpu_sets(ev, probe, block, tau, rows):
+    import torch
+    cfg = probe.cfg
+    q, k, v = to_device(probe)
+    keep, uni, ws = ev.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                        block, tau)
+    torch.cuda.synchronize()
+    assert ev.evisel_status(ws) == 0
+    bits = keep[:, :, torch.as_tensor(rows, device="cuda")].cpu().numpy().view(np.uint32)   # [hq, W, len(rows)]
+    ws.free()
+    sets = {}
+    for h in range(bits.shape[0]):
+        for r, row in enumerate(rows):
+            ids = [w * 32 + j for w in range(bits.shape[1]) for j in range(32) if (int(bits[h, w, r]) >> j) & 1]
+            sets[(h, int(row))] = ids
+    return sets, keep, uni
+
+
+def _check_sets(gpu, probs, cu, n_vis, block, tau, label):
+    cu = np.asarray(cu)
+    for (h, row), ids in gpu.items():
+        hist, p = probs[(h, row)]
+        b = int(np.searchsorted(cu, row, side="right") - 1)
+        pos = row - int(cu[b])
+        nv = int(n_vis[b])
+        own = pos // block if pos < nv else nv // block + (pos - nv) // block
+        assert own in ids, (label, h, row, "own block")
+        s = [j for j in ids if j != own]
+        assert set(s) <= set(int(x) for x in hist), (label, h, row, "outside H_i")
+        if hist.size == 0:
+            assert not s
+            continue
+        kept = np.isin(hist, s)
+        mass = p[kept].sum()
+        assert mass >= tau - EPS, (label, h, row, "mass", mass)
+        assert mass - p[kept].min() < tau + EPS, (label, h, row, "not minimal", mass, p[kept].min())
+        if (~kept).any():
+            # top set, up to the builder's resolution: log2 p within (max - min) / 16384 of each other may tie
+            lp = np.log2(p[p > 0])
+            res = (lp.max() - lp.min()) / 16384 + LOG2_EPS
+            assert np.log2(p[kept].min()) >= np.log2(p[~kept].max()) - res, (label, h, row, "not a top set")
+
+
+def _all_rows(probe):
+    return np.arange(int(probe.cu_seqlens[-1]))
+
+
+@pytest.mark.parametrize("name,block,tau", [("tiny", 16, 0.97), ("single", 16, 0.97), ("single", 16, 0.5)])
+def test_topp_sets_small(cuda_lib, name, block, tau):
+    probe = wl.make_probe(wl.CONFIGS[name])
+    rows = _all_rows(probe)
+    gpu, _, _ = _gpu_sets(cuda_lib, probe, block, tau, rows)
+    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, tau, rows=rows,
+                                      kbar_round="bf16")
+    _check_sets(gpu, probs, probe.cu_seqlens, probe.n_vis, block, tau, name)
+
+
+@pytest.mark.parametrize("name,block,n_rows", [("long65k", 64, 24), ("varlen8", 16, 24)])
+def test_topp_sets_sampled(cuda_lib, name, block, n_rows):
+    probe = wl.make_probe(wl.CONFIGS[name])
+    rng = np.random.default_rng(3)
+    n = int(probe.cu_seqlens[-1])
+    rows = np.unique(np.concatenate([[0, n - 1], probe.cu_seqlens[1:-1], rng.integers(0, n, n_rows)]))
+    gpu, _, _ = _gpu_sets(cuda_lib, probe, block, 0.97, rows)
+    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, 0.97, rows=rows,
+                                      kbar_round="bf16")
+    _check_sets(gpu, probs, probe.cu_seqlens, probe.n_vis, block, 0.97, name)
+
+
+EDGE = {
+    "planted_sharp_b32": dict(frames=(40,), n_text=(60,), npf=64, hq=4, hkv=2, d=128, tile=128, window=2, sharp=True),
+    "t64_d64_b16": dict(frames=(20,), n_text=(40,), hq=6, hkv=2, d=64, tile=64, window=2),
+    "varlen_mixed": dict(frames=(3, 0, 17, 8), n_text=(12, 40, 0, 130), hq=4, hkv=2, d=128, tile=128, window=2),
+}
+
+
+@pytest.mark.parametrize("name,block,tau", [("planted_sharp_b32", 32, 0.97), ("planted_sharp_b32", 64, 0.3),
+                                            ("t64_d64_b16", 16, 0.9), ("varlen_mixed", 16, 0.97),
+                                            ("varlen_mixed", 16, 1.0)])
+def test_topp_edge_cases(cuda_lib, name, block, tau):
+    from test_gpu_parity import _custom
+    probe = _custom(**EDGE[name])
+    rows = _all_rows(probe)
+    gpu, _, _ = _gpu_sets(cuda_lib, probe, block, tau, rows)
+    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, tau, rows=rows,
+                                      kbar_round="bf16")
+    _check_sets(gpu, probs, probe.cu_seqlens, probe.n_vis, block, min(tau, 1.0 - 1e-6), name)
+
+
+def test_topp_union_drives_the_probe(cuda_lib):
+    """The tile union equals the union of the GPU's own sets; as a mask it runs the probe."""
+    import torch
+    probe = wl.make_probe(wl.CONFIGS["single"])
+    cfg = probe.cfg
+    rows = _all_rows(probe)
+    gpu, keep, uni = _gpu_sets(cuda_lib, probe, 16, 0.5, rows)
+    row_ptr, col_idx = B.tile_union_to_csr(uni, probe.n_vis, cfg.tile)
+    # union of the sets of every visual row and head, mapped to key tiles
+    n_vis = int(probe.n_vis[0])
+    bpt = cfg.tile // 16
+    n_vt = -(-n_vis // cfg.tile)
+    want = [set() for _ in range(n_vt)]
+    for (h, row), ids in gpu.items():
+        if row < n_vis:
+            want[row // cfg.tile] |= {j // bpt for j in ids if j < n_vis // 16}
+    for r in range(n_vt):
+        assert sorted(want[r]) == list(col_idx[row_ptr[r]:row_ptr[r + 1]]), r
+    # the probe with this mask
+    q, k, v = to_device(probe)
+    o, lse, ws = cuda_lib.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame,
+                                                 cfg.tile, row_ptr, col_idx)
+    torch.cuda.synchronize()
+    ws.free()
+    pick = np.array([0, 100, 1000, 2047, 4095, 4100, 4159])
+    o_ref, lse_ref = oracle.probe_rows(probe.q, probe.k, probe.v, probe.cu_seqlens, probe.n_vis, cfg.tile, row_ptr,
+                                       col_idx, pick)
+    check_o(o.float().cpu().numpy()[pick], o_ref, "probe on the top-p union")
+    check_lse(lse.cpu().numpy()[:, pick], lse_ref, "probe on the top-p union")

@@ -13,7 +13,8 @@ Each test names the pin it realises:
   O9  planted frames rank top on the head-summed frame map
   O10 linearity of O in V
   F1-F4 the intra-frame cue A_if (closed form, dense weights, brute force, structure)
-  H1-H5 top-p block retention (closed form, brute force, planted block, limits, keep-all)
+  H1-H6 top-p block retention (closed form, brute force, planted block, limits, keep-all,
+        bf16 rounding of the block means)
   G1-G5 the cross-frame cue A_ff and E_ff (closed form, mass balance with A_if, brute force,
         dense weights, a hand-worked E_ff)
 """
@@ -720,3 +721,12 @@ def test_H3_catches_an_ascending_order(monkeypatch):
     monkeypatch.setattr(ot, "select_prefix", ascending)
     with pytest.raises(AssertionError):
         test_H3_topp_planted_block_takes_the_mass()
+
+
+def test_H6_round_bf16_matches_torch():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(47)
+    x = np.concatenate([rng.standard_normal(4096).astype(np.float32) * 10 ** rng.uniform(-6, 6, 4096),
+                        np.array([1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -(1.0 + 2 ** -8)], np.float32)])
+    from oracle.topp import round_bf16
+    np.testing.assert_array_equal(round_bf16(x), torch.from_numpy(x).to(torch.bfloat16).double().numpy())
