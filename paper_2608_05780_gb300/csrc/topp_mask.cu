@@ -245,85 +245,101 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
         for (int ch = 0; ch < n_ch; ++ch) {
           const int t = (hh * kPasses + pass) * n_ch + ch, b = t % 2;
           ok = ok && warp_wait(bar(C::B_SF + b), (t / 2) & 1, abort_flag);
-          uint32_t bits[4] = {0u, 0u, 0u, 0u};
           int run_bin = -1;                        // histogram passes: consecutive keys of one bin add in a register
           float run = 0.f;
           if (ok && __any_sync(0xffffffffu, nh > ch * kCols)) {   // warp-uniform: tcgen05.ld is collective
             ptx::tc_fence_after();
-#pragma unroll
+            // One compact loop per pass (uniform over the warp), 32 columns at a time.
+#pragma unroll 1
             for (int c0 = 0; c0 < kCols; c0 += 32) {
               uint32_t r[32];
               ptx::tmem_ld32(tbase + b * kCols + c0, r);
               ptx::tmem_wait_ld();
-              float cmax = -INFINITY;
+              const int jn = nh - (ch * kCols + c0);         // columns e < jn are in H_i
               if (pass == 0) {
+                float cmax = -INFINITY;
 #pragma unroll
-                for (int e = 0; e < 32; ++e)
-                  if (ch * kCols + c0 + e < nh) {
-                    const float x = __uint_as_float(r[e]) * sc;
+                for (int e = 0; e < 32; ++e) {
+                  const float x = __uint_as_float(r[e]) * sc;
+                  if (e < jn) {
                     cmax = fmaxf(cmax, x);
                     gmin = fminf(gmin, x);
                   }
+                }
                 if (cmax > m) {
                   z = (m == -INFINITY) ? 0.f : z * ptx::ex2(m - cmax);
                   m = cmax;
                 }
-              }
+                float zs = 0.f;
 #pragma unroll
-              for (int e = 0; e < 32; ++e) {
-                const int j = ch * kCols + c0 + e;
-                if (j >= nh) continue;
-                const float x = __uint_as_float(r[e]) * sc;
-                const float w = ptx::ex2(x - m);
-                if (pass == 0) {
-                  z += w;
-                  continue;
-                }
-                const float u = m - x;                     // >= 0: distance below the max
-                const int bin1 = min(kBins - 1, static_cast<int>(u * inv_w1));
-                if (pass == 1) {
+                for (int e = 0; e < 32; ++e)
+                  if (e < jn) zs += ptx::ex2(__uint_as_float(r[e]) * sc - m);
+                z += zs;
+              } else if (pass == 1) {
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                  if (e >= jn) break;
+                  const float x = __uint_as_float(r[e]) * sc;
+                  const int bin1 = min(kBins - 1, static_cast<int>((m - x) * inv_w1));
                   if (bin1 != run_bin) {
                     if (run_bin >= 0) hist[run_bin * kRows] += run;
                     run_bin = bin1;
                     run = 0.f;
                   }
-                  run += w;
-                  continue;
+                  run += ptx::ex2(x - m);
                 }
-                const int bin2 = bin1 == b1 ? min(kBins - 1, static_cast<int>((u - b1 * w1) * inv_w2)) : 0;
-                if (pass == 2) {
-                  if (bin1 == b1) {
-                    if (bin2 != run_bin) {
-                      if (run_bin >= 0) hist[run_bin * kRows] += run;
-                      run_bin = bin2;
-                      run = 0.f;
-                    }
-                    run += w;
+              } else if (pass == 2) {
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                  if (e >= jn) break;
+                  const float x = __uint_as_float(r[e]) * sc;
+                  const float u = m - x;
+                  if (min(kBins - 1, static_cast<int>(u * inv_w1)) != b1) continue;
+                  const int bin2 = min(kBins - 1, static_cast<int>((u - b1 * w1) * inv_w2));
+                  if (bin2 != run_bin) {
+                    if (run_bin >= 0) hist[run_bin * kRows] += run;
+                    run_bin = bin2;
+                    run = 0.f;
                   }
-                  continue;
+                  run += ptx::ex2(x - m);
                 }
-                bool kept = bin1 < b1 || (bin1 == b1 && bin2 < b2);
-                if (bin1 == b1 && bin2 == b2) {                 // ties: lower ids first
-                  kept = above2 + tie < target;
-                  tie += w;
+              } else {
+                uint32_t word = 0u;
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                  if (e >= jn) break;
+                  const float x = __uint_as_float(r[e]) * sc;
+                  const float u = m - x;
+                  const int bin1 = min(kBins - 1, static_cast<int>(u * inv_w1));
+                  bool kept = bin1 < b1;
+                  if (bin1 == b1) {
+                    const int bin2 = min(kBins - 1, static_cast<int>((u - b1 * w1) * inv_w2));
+                    kept = bin2 < b2;
+                    if (bin2 == b2) {                             // ties: lower ids first
+                      kept = above2 + tie < target;
+                      tie += ptx::ex2(x - m);
+                    }
+                  }
+                  if (kept) word |= 1u << e;
                 }
-                if (kept) bits[(c0 + e) >> 5] |= 1u << ((c0 + e) & 31);
+                const int w = ch * 4 + (c0 >> 5);
+                if (row_ok && w < L.n_words) {
+                  if (w == nh >> 5) word |= 1u << (nh & 31);     // the row's own block
+                  keep[static_cast<int64_t>(w) * L.n_tok] = word;
+                }
               }
             }
             ptx::tc_fence_before();
-          }
-          ptx::mbar_arrive(bar(C::B_SE + b));
-          if (run_bin >= 0) hist[run_bin * kRows] += run;
-          if (pass == 3 && row_ok && ok) {
-#pragma unroll
+          } else if (pass == 3 && row_ok && ok) {
+            // No column of this chunk is in H_i for the warp: zeros (and the own block).
             for (int wi = 0; wi < 4; ++wi) {
               const int w = ch * 4 + wi;
               if (w >= L.n_words) break;
-              uint32_t word = bits[wi];
-              if (w == nh >> 5) word |= 1u << (nh & 31);   // the row's own block
-              keep[static_cast<int64_t>(w) * L.n_tok] = word;
+              keep[static_cast<int64_t>(w) * L.n_tok] = w == nh >> 5 ? 1u << (nh & 31) : 0u;
             }
           }
+          ptx::mbar_arrive(bar(C::B_SE + b));
+          if (run_bin >= 0) hist[run_bin * kRows] += run;
         }
         // Between passes: the bin widths and the boundary (bin, mass above it).
         // A boundary is the first bin whose cumulative mass from the top reaches
