@@ -102,6 +102,16 @@ typedef struct {
                                     q and k (no spill; q and k, like lse, must stay
                                     alive until evisel_evidence_reduce() ran). Same
                                     outputs within fp32 rounding. */
+  const uint32_t* keep;          /* NULL, or device per-row block masks from
+                                    evisel_topp_mask(): row i of head h attends only
+                                    the keys of blocks whose bit is set (its top-p
+                                    set S_i and its own block, causally), within the
+                                    kv tiles the mask above keeps (pass the row
+                                    tiles' union). Not with cross_frame or
+                                    text_evidence; evisel_intra_frame_evidence and
+                                    evisel_cross_frame_evidence refuse such a probe. */
+  int32_t keep_words;            /* W of keep [hq, W, N_tot]                        */
+  int32_t keep_block;            /* the block size B the masks were built with      */
 } evisel_probe_args;
 
 /* Block-sparse causal GQA varlen attention (Eq. 1; Appendix Eq. 8 and Eq. 11

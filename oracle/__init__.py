@@ -23,5 +23,5 @@ from .attention import (  # noqa: F401
     cross_frame, e_ff,
 )
 from .topp import (  # noqa: F401
-    block_layout, block_means, select_prefix, retained_blocks, attended_mask, probe_rows_topp,
+    block_layout, block_means, select_prefix, retained_blocks, attended_mask, probe_rows_topp, evidence_topp,
 )

@@ -143,3 +143,45 @@ def probe_rows_topp(q, k, v, cu_seqlens, n_vis, block, kept, rows, scale=None):
             lse[h, r] = mx + math.log(w.sum())
             o[r, h, :] = (w / w.sum()) @ v[s0:s1, h // gq, :].astype(np.float64)
     return o, lse
+
+
+def evidence_topp(q, k, cu_seqlens, n_vis, tokens_per_frame, block, kept, scale=None):
+    """The evidence maps of the text rows attending to their retained blocks
+    ``kept`` ({(h, row): block ids}) and their own block's causal prefix:
+    P_im = exp(s_im - LSE_i) over the attended keys, summed over the text rows
+    into tok [Hq, sum n_vis], then frame [Hq, sum T], head [B, Hq] and
+    aqf [sum T] as in the dense evidence (Sec. 3.2)."""
+    q = np.asarray(q); k = np.asarray(k)
+    n, hq, d = q.shape
+    gq = hq // k.shape[1]
+    scale = 1.0 / math.sqrt(d) if not scale else float(scale)
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    n_vis = np.asarray(n_vis, dtype=np.int64)
+    npf = int(tokens_per_frame)
+    frames = n_vis // npf
+    vis_off = np.concatenate([[0], np.cumsum(n_vis)])
+    fr_off = np.concatenate([[0], np.cumsum(frames)])
+    tok = np.zeros((hq, int(vis_off[-1])))
+    frame = np.zeros((hq, int(fr_off[-1])))
+    head = np.zeros((len(n_vis), hq))
+    aqf = np.zeros(int(fr_off[-1]))
+    for b in range(len(n_vis)):
+        s0, s1, nv = int(cu[b]), int(cu[b + 1]), int(n_vis[b])
+        n_text = s1 - s0 - nv
+        for h in range(hq):
+            t_map = np.zeros(nv)
+            for row in range(s0 + nv, s1):
+                m = attended_mask(row - s0, nv, n_text, block, kept[(h, row)])
+                s = scale * (k[s0:s1, h // gq, :].astype(np.float64) @ q[row, h, :].astype(np.float64))
+                s = np.where(m, s, -np.inf)
+                mx = s.max()
+                p = np.exp(s - mx)
+                p /= p.sum()
+                t_map += p[:nv]
+            tok[h, vis_off[b]:vis_off[b + 1]] = t_map
+            f_map = t_map.reshape(int(frames[b]), npf).sum(axis=1)
+            frame[h, fr_off[b]:fr_off[b + 1]] = f_map
+            head[b, h] = f_map.sum()
+        if n_text > 0:
+            aqf[fr_off[b]:fr_off[b + 1]] = frame[:, fr_off[b]:fr_off[b + 1]].sum(axis=0) / (hq * n_text)
+    return tok, frame, head, aqf

@@ -46,6 +46,9 @@ class ProbeArgs(ctypes.Structure):
         ("lse", ctypes.c_void_p),
         ("cross_frame", ctypes.c_int32),
         ("text_evidence", ctypes.c_int32),
+        ("keep", ctypes.c_void_p),
+        ("keep_words", ctypes.c_int32),
+        ("keep_block", ctypes.c_int32),
     ]
 
 
@@ -132,7 +135,7 @@ class Workspace:
 
 
 def make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
-              softmax_scale=0.0, cross_frame=False, text_evidence=False):
+              softmax_scale=0.0, cross_frame=False, text_evidence=False, keep=None, keep_block=0):
     """Fills the C struct; returns (struct, keepalive) - keepalive holds the host arrays."""
     cu, cu_p = _i32(cu_seqlens)
     nv, nv_p = _i32(n_vis)
@@ -154,16 +157,22 @@ def make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_i
     a.o, a.lse = o.data_ptr(), lse.data_ptr()
     a.cross_frame = int(bool(cross_frame))
     a.text_evidence = int(bool(text_evidence))
+    if keep is not None:
+        a.keep = keep.data_ptr()
+        a.keep_words = int(keep.shape[1])
+        a.keep_block = int(keep_block)
     return a, (cu, nv, rp, ci)
 
 
 def evisel_probe_attention(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx,
                            ws=None, o=None, lse=None, softmax_scale=0.0, stream=None, cross_frame=False,
-                           text_evidence=False):
+                           text_evidence=False, keep=None, keep_block=0):
     """Block-sparse GQA varlen probe attention. q/k/v: CUDA bf16 [N, H, d].
     ``cross_frame`` also keeps the partials evisel_cross_frame_evidence reads;
     ``text_evidence`` makes evisel_evidence_reduce recompute the text-row
-    probabilities from q and k instead of spilling the logits.
+    probabilities from q and k instead of spilling the logits; ``keep`` (from
+    evisel_topp_mask, with its ``keep_block``) restricts every row to its
+    retained blocks.
 
     Returns (o [N, hq, d] bf16, lse [hq, N] fp32, ws).
     """
@@ -180,7 +189,7 @@ def evisel_probe_attention(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, r
     if ws is None:
         ws = Workspace()
     args, keep = make_args(q, k, v, cu_seqlens, n_vis, tokens_per_frame, tile, row_ptr, col_idx, o, lse,
-                           softmax_scale, cross_frame, text_evidence)
+                           softmax_scale, cross_frame, text_evidence, keep, keep_block)
     _check(lib.evisel_probe_attention(ctypes.byref(args), _stream_handle(stream), ctypes.byref(ws.ptr)))
     del keep
     return o, lse, ws

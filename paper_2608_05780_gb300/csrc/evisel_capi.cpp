@@ -104,6 +104,20 @@ int validate(const evisel_probe_args* a) {
     return fail(EVISEL_EINVAL, "softmax_scale must be finite and >= 0");
   if (a->cross_frame != 0 && a->cross_frame != 1) return fail(EVISEL_EINVAL, "cross_frame must be 0 or 1");
   if (a->text_evidence != 0 && a->text_evidence != 1) return fail(EVISEL_EINVAL, "text_evidence must be 0 or 1");
+  if (a->keep) {
+    const int kb = a->keep_block;
+    if (kb < 16 || kb > npf || (kb & (kb - 1)) != 0)
+      return fail(EVISEL_EUNSUPPORTED, "keep_block must be a power of two in [16, tokens_per_frame]");
+    if (a->cross_frame || a->text_evidence)
+      return fail(EVISEL_EUNSUPPORTED, "per-row block masks do not combine with cross_frame or text_evidence");
+    if (reinterpret_cast<uintptr_t>(a->keep) & 3u) return fail(EVISEL_EINVAL, "keep must be 4-byte aligned");
+    int max_blocks = 0;
+    for (int b = 0; b < a->num_videos; ++b) {
+      const int nv = a->n_vis_h[b], nt = a->cu_seqlens_h[b + 1] - a->cu_seqlens_h[b] - nv;
+      max_blocks = std::max(max_blocks, nv / kb + (nt + kb - 1) / kb);
+    }
+    if (a->keep_words < (max_blocks + 31) / 32) return fail(EVISEL_EINVAL, "keep_words too small for the blocks");
+  }
   if (a->cross_frame && npf < 16)
     return fail(EVISEL_EUNSUPPORTED, "cross-frame partials need tokens_per_frame >= 16");
   if (a->num_videos == 0) return EVISEL_OK;
@@ -360,6 +374,7 @@ struct evisel_ws {
   // last probe, for the evidence pass
   bool probed = false;
   const float* lse = nullptr;
+  bool probe_keep = false;          // the last probe ran with per-row block masks
   const void* q = nullptr;          // the probe's q and k (read by the recompute evidence)
   const void* k = nullptr;
   int hkv = 0, head_dim = 0;
@@ -551,6 +566,11 @@ int evisel_probe_attention(const evisel_probe_args* args, void* stream_ptr, evis
     L.tile = args->tile;
     L.scale = scale;
     L.scale_log2 = scale * 1.4426950408889634f;
+    if (args->keep) {
+      L.keep = args->keep;
+      L.keep_words = args->keep_words;
+      L.keep_block = args->keep_block;
+    }
     if (P.cross_frame && P.nnz_vis > 0) {
       L.fspill = ws->d_fspill;
       L.fs_nnz = P.nnz_vis;
@@ -576,6 +596,7 @@ int evisel_probe_attention(const evisel_probe_args* args, void* stream_ptr, evis
     }
   }
   ws->probed = true;
+  ws->probe_keep = args->keep != nullptr;
   ws->lse = args->lse;
   ws->q = args->q;
   ws->k = args->k;
@@ -659,6 +680,7 @@ int evisel_intra_frame_evidence(const evisel_probe_args* args, const evisel_ws* 
   int rc = validate(args);
   if (rc != EVISEL_OK) return rc;
   if (!ws->probed || !ws->have_plan) return fail(EVISEL_ESTATE, "no probe has run on this workspace");
+  if (ws->probe_keep) return fail(EVISEL_EUNSUPPORTED, "the probe ran with per-row block masks");
   const Plan& P = ws->plan;
   if (static_cast<int>(P.videos.size()) != args->num_videos)
     return fail(EVISEL_EINVAL, "args do not match the probe that ran on this workspace");
@@ -708,6 +730,7 @@ int evisel_cross_frame_evidence(const evisel_probe_args* args, evisel_ws* ws, fl
   if (!ws->probed || !ws->have_plan) return fail(EVISEL_ESTATE, "no probe has run on this workspace");
   const Plan& P = ws->plan;
   if (!P.cross_frame) return fail(EVISEL_ESTATE, "the probe on this workspace ran without cross_frame");
+  if (ws->probe_keep) return fail(EVISEL_EUNSUPPORTED, "the probe ran with per-row block masks");
   if (static_cast<int>(P.videos.size()) != args->num_videos || plan_key(args) != ws->key)
     return fail(EVISEL_EINVAL, "args do not match the probe that ran on this workspace");
   if (P.aff_floats > 0 && !aff) return fail(EVISEL_EINVAL, "aff is NULL");

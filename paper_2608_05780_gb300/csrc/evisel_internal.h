@@ -94,6 +94,10 @@ struct ProbeLaunch {
   // partial (a key frame is N_v / fs_span consecutive spans).
   float* fspill;
   int fs_nnz, fs_span;
+  // Per-row block masks (null: the tile mask alone): keep[h][word][row], bit j
+  // of word w = block 32 w + j of the row's video, blocks of keep_block tokens.
+  const uint32_t* keep;
+  int keep_words, keep_block;
 };
 
 struct CombineLaunch {

@@ -179,6 +179,8 @@ extern "C" int evisel_probe_evidence_noalloc(const evisel_probe_args* args, floa
   if (rc != EVISEL_OK) return rc;
   if (args->cross_frame)
     return set_last_error(EVISEL_EUNSUPPORTED, "cross-frame partials need a workspace (evisel_probe_attention)");
+  if (args->keep)
+    return set_last_error(EVISEL_EUNSUPPORTED, "per-row block masks need a workspace (evisel_probe_attention)");
   Counts c;
   make_plan(args, c, nullptr);
   if ((c.total_vis > 0 && (!tok || !frame)) || (args->num_videos > 0 && !head) || (c.total_frames > 0 && !aqf))

@@ -346,7 +346,7 @@ __device__ __forceinline__ void mma_issuer(const ProbeLaunch& L, const WorkItem&
   __syncwarp();
 }
 
-template <int TILE, int D, int NS, int FSW>
+template <int TILE, int D, int NS, int FSW, int EMB>
 __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const WorkItem& it, int slot, uint32_t sbase,
                                                  uint32_t tmem_base, volatile int* abort_flag) {
   using C = Cfg<TILE, D, NS>;
@@ -393,6 +393,18 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
       fs_row = L.fspill + (static_cast<int64_t>(head) * L.fs_nnz + it.kv_begin) * (TILE / FSW) * TILE + row_local;
   }
 
+  // Per-row block masks (EMB = their block size; 0: none): the row's bit per
+  // block of its video (top-p retention and the own block), applied to the
+  // keys of every kv tile before the max, the spill and P.
+  [[maybe_unused]] const uint32_t* em_row = nullptr;
+  [[maybe_unused]] int em_vis_start = 0, em_n_vis = 0;
+  if constexpr (EMB > 0) {
+    const VideoInfo evi = L.videos[it.video];
+    em_vis_start = evi.vis_start;
+    em_n_vis = evi.n_vis;
+    if (row_ok) em_row = L.keep + static_cast<int64_t>(head) * L.keep_words * L.n_tok + qpos;
+  }
+
   float m_used = -INFINITY;   // running max, log2 units
   float l_sum = 0.f;
   bool ok = true;
@@ -414,6 +426,23 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
     }
     const bool spill = spill_rows && kv.visual;
     float* spill_dst = spill ? spill_row + static_cast<int64_t>(kv.start - vis_start) * 32 : nullptr;
+    [[maybe_unused]] uint32_t em_bits = 0xffffffffu;   // bit q: the tile's q-th block is attended
+    if constexpr (EMB > 0) {
+      if (em_row) {
+        const int blk0 = kv.visual ? (kv.start - em_vis_start) / EMB
+                                   : em_n_vis / EMB + (kv.start - em_vis_start - em_n_vis) / EMB;
+        em_bits = em_row[static_cast<int64_t>(blk0 >> 5) * L.n_tok] >> (blk0 & 31);
+      }
+    }
+    auto apply_em = [&](float* sv, int h) {
+      if constexpr (EMB > 0) {
+        if ((em_bits & ((1u << (TILE / EMB)) - 1u)) != (1u << (TILE / EMB)) - 1u) {
+#pragma unroll
+          for (int c = 0; c < 64; ++c)
+            if (!((em_bits >> ((h * 64 + c) / EMB)) & 1u)) sv[c] = -INFINITY;
+        }
+      }
+    };
 
     // Pass 1: row max (and the text rows' logit spill), 64 columns at a time.
     float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
@@ -431,6 +460,7 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
           s[32 + e] = __uint_as_float(r1[e]);
         }
       }
+      apply_em(s, h);
       if (spill) {
         float* dst = spill_dst + h * 64 * 32;
 #pragma unroll
@@ -504,6 +534,7 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
           s[32 + e] = __uint_as_float(r1[e]);
         }
       }
+      apply_em(s, h);
       if (limit < TILE) {
 #pragma unroll
         for (int c = 0; c < 64; ++c) s[c] = h * 64 + c < limit ? s[c] : -INFINITY;
@@ -638,7 +669,7 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
   }
 }
 
-template <int TILE, int D, int NS, int FSW>
+template <int TILE, int D, int NS, int FSW, int EMB>
 __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_constant__ ProbeLaunch L) {
   using C = Cfg<TILE, D, NS>;
   extern __shared__ uint8_t smem_raw[];
@@ -673,7 +704,7 @@ __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_co
   } else if (warp == kWarpMma) {
     mma_issuer<TILE, D, NS>(L, it, sbase, tmem, abort_flag);
   } else {
-    softmax_epilogue<TILE, D, NS, FSW>(L, it, warp / 4, sbase, tmem, abort_flag);
+    softmax_epilogue<TILE, D, NS, FSW, EMB>(L, it, warp / 4, sbase, tmem, abort_flag);
   }
   ptx::tc_fence_before();
   __syncthreads();
@@ -683,11 +714,11 @@ __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_co
   }
 }
 
-template <int TILE, int D, int FSW>
+template <int TILE, int D, int FSW, int EMB = 0>
 cudaError_t launch_cfg(const ProbeLaunch& L, cudaStream_t stream) {
   constexpr int NS = 2;
   using C = Cfg<TILE, D, NS>;
-  auto kern = probe_attn_kernel<TILE, D, NS, FSW>;
+  auto kern = probe_attn_kernel<TILE, D, NS, FSW, EMB>;
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
@@ -702,6 +733,18 @@ cudaError_t launch_cfg(const ProbeLaunch& L, cudaStream_t stream) {
 // key spans of fsw tokens (16, 32 or 64).
 template <int TILE, int D>
 cudaError_t launch_fsw(const ProbeLaunch& L, int fsw, cudaStream_t stream) {
+  if (L.keep) {                                  // per-row block masks (not with cross-frame partials)
+    if (fsw != 0) return cudaErrorInvalidValue;
+    switch (L.keep_block) {
+      case 16: return launch_cfg<TILE, D, 0, 16>(L, stream);
+      case 32: return launch_cfg<TILE, D, 0, 32>(L, stream);
+      case 64: return launch_cfg<TILE, D, 0, 64>(L, stream);
+      case 128:
+        if constexpr (TILE == 128) return launch_cfg<TILE, D, 0, 128>(L, stream);
+        return cudaErrorInvalidValue;
+      default: return cudaErrorInvalidValue;
+    }
+  }
   switch (fsw) {
     case 0: return launch_cfg<TILE, D, 0>(L, stream);
     case 16: return launch_cfg<TILE, D, 16>(L, stream);

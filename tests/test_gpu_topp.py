@@ -143,3 +143,70 @@ def test_topp_union_drives_the_probe(cuda_lib):
                                        col_idx, pick)
     check_o(o.float().cpu().numpy()[pick], o_ref, "probe on the top-p union")
     check_lse(lse.cpu().numpy()[:, pick], lse_ref, "probe on the top-p union")
+
+
+def _sets_from_keep(keep, rows, cu, n_vis, block):
+    """{(h, row): retained block ids} without the own block, from keep bits."""
+    import torch
+    bits = keep[:, :, torch.as_tensor(rows, device=keep.device)].cpu().numpy().view(np.uint32)
+    out = {}
+    cu = np.asarray(cu)
+    for h in range(bits.shape[0]):
+        for r, row in enumerate(rows):
+            b = int(np.searchsorted(cu, row, side="right") - 1)
+            pos = int(row) - int(cu[b])
+            nv = int(n_vis[b])
+            own = pos // block if pos < nv else nv // block + (pos - nv) // block
+            ids = [w * 32 + j for w in range(bits.shape[1]) for j in range(32) if (int(bits[h, w, r]) >> j) & 1]
+            out[(h, int(row))] = [j for j in ids if j != own]
+    return out
+
+
+@pytest.mark.parametrize("name,block,tau", [("single", 16, 0.5), ("tiny", 16, 0.6)])
+def test_probe_attends_only_the_retained_blocks(cuda_lib, name, block, tau):
+    """Probe with the per-row masks (and the union as the tile mask) against the
+    oracle restricted to the same sets: O, LSE and the evidence maps."""
+    import torch
+    from gpu_helpers import check_maps, np32
+    probe = wl.make_probe(wl.CONFIGS[name])
+    cfg = probe.cfg
+    q, k, v = to_device(probe)
+    keep, uni, ws = cuda_lib.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                              block, tau)
+    row_ptr, col_idx = B.tile_union_to_csr(uni, probe.n_vis, cfg.tile)
+    o, lse, ws = cuda_lib.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame,
+                                                 cfg.tile, row_ptr, col_idx, ws=ws, keep=keep, keep_block=block)
+    maps = cuda_lib.evisel_evidence_reduce(ws, cfg.hq, probe.n_vis, cfg.tokens_per_frame, len(probe.n_vis))
+    torch.cuda.synchronize()
+    assert cuda_lib.evisel_status(ws) == 0
+    n = int(probe.cu_seqlens[-1])
+    rows = np.arange(n)
+    kept = _sets_from_keep(keep, rows, probe.cu_seqlens, probe.n_vis, block)
+    pick = np.unique(np.concatenate([np.arange(0, n, max(1, n // 40)), np.arange(n - 8, n)]))
+    o_ref, lse_ref = oracle.probe_rows_topp(probe.q, probe.k, probe.v, probe.cu_seqlens, probe.n_vis, block, kept,
+                                            pick)
+    check_o(o.float().cpu().numpy()[pick], o_ref, f"{name} top-p probe")
+    check_lse(lse.cpu().numpy()[:, pick], lse_ref, f"{name} top-p probe")
+    want = oracle.evidence_topp(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, block, kept)
+    check_maps([np32(m) for m in maps], list(want), probe, label=f"{name} top-p evidence")
+    ws.free()
+
+
+def test_keep_refused_where_it_does_not_apply(cuda_lib):
+    import torch
+    probe = wl.make_probe(wl.CONFIGS["tiny"])
+    cfg = probe.cfg
+    q, k, v = to_device(probe)
+    keep, uni, ws = cuda_lib.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                              16, 0.9)
+    row_ptr, col_idx = B.tile_union_to_csr(uni, probe.n_vis, cfg.tile)
+    with pytest.raises(B.EviselError):
+        cuda_lib.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                        row_ptr, col_idx, ws=ws, keep=keep, keep_block=16, cross_frame=True)
+    o, lse, ws = cuda_lib.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame,
+                                                 cfg.tile, row_ptr, col_idx, ws=ws, keep=keep, keep_block=16)
+    with pytest.raises(B.EviselError):
+        cuda_lib.evisel_intra_frame_evidence(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                             row_ptr, col_idx, o, lse, ws)
+    torch.cuda.synchronize()
+    ws.free()

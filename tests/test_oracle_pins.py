@@ -13,8 +13,8 @@ Each test names the pin it realises:
   O9  planted frames rank top on the head-summed frame map
   O10 linearity of O in V
   F1-F4 the intra-frame cue A_if (closed form, dense weights, brute force, structure)
-  H1-H6 top-p block retention (closed form, brute force, planted block, limits, keep-all,
-        bf16 rounding of the block means)
+  H1-H7 top-p block retention (closed form, brute force, planted block, limits, keep-all,
+        bf16 rounding of the block means, evidence with every block kept)
   G1-G5 the cross-frame cue A_ff and E_ff (closed form, mass balance with A_if, brute force,
         dense weights, a hand-worked E_ff)
 """
@@ -730,3 +730,12 @@ def test_H6_round_bf16_matches_torch():
                         np.array([1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -(1.0 + 2 ** -8)], np.float32)])
     from oracle.topp import round_bf16
     np.testing.assert_array_equal(round_bf16(x), torch.from_numpy(x).to(torch.bfloat16).double().numpy())
+
+
+def test_H7_evidence_with_every_block_kept_is_the_dense_evidence():
+    c = _topp_case(48, videos=((16, 6), (12, 5)))
+    sets, _ = oracle.retained_blocks(c["q"], c["k"], c["cu"], c["n_vis"], 4, 1.0 - 1e-12)
+    got = oracle.evidence_topp(c["q"], c["k"], c["cu"], c["n_vis"], 4, 4, sets)
+    want = oracle.evidence(c["q"], c["k"], c["cu"], c["n_vis"], 4)
+    for g, w in zip(got, want):
+        np.testing.assert_allclose(g, w, atol=1e-13)
