@@ -463,6 +463,16 @@ def bench_ours(args, cfg):
         ev.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, npf, 0.97, ws=ws_tp)
 
     tp_ms = _time(topp)
+    # the probe restricted to each row's retained blocks: the row tiles' union
+    # as the tile mask, the per-row bits inside
+    tp_row_ptr, tp_col_idx = ev.tile_union_to_csr(uni_tp, probe.n_vis, cfg.tile)
+    tp_args = (q, k, v, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, tp_row_ptr, tp_col_idx)
+
+    def probe_topp():
+        ev.evisel_probe_attention(*tp_args, ws=ws_tp, o=o_cf, lse=lse_cf, keep=keep_tp, keep_block=npf)
+
+    tpp_ms = _time(probe_topp)
+    tp_tiles = int(tp_row_ptr[-1])
     status = ev.evisel_status(ws_tp)
     ws_tp.free()
     del keep_tp, uni_tp
@@ -502,7 +512,9 @@ def bench_ours(args, cfg):
                                 "frac_of_hbm": if_bytes / (if_ms * 1e-3) / 1e9 / peaks["hbm"], "bytes": if_bytes,
                                 "tflops": if_flop / (if_ms * 1e-3) / 1e12},
                 "topp_mask": {"ms": tp_ms, "block": npf, "tau_p": 0.97, "blocks": n_blk,
-                              "tflops_history": tp_flop / (tp_ms * 1e-3) / 1e12},
+                              "tflops_history": tp_flop / (tp_ms * 1e-3) / 1e12,
+                              "probe_ms": tpp_ms, "union_tiles": tp_tiles,
+                              "static_mask_tiles": int(probe.row_ptr[-1])},
                 "text_evidence_recompute": {"step_ms": te_step_ms, "probe_ms": te_probe_ms, "evidence_ms": te_ev_ms,
                                             "tflops": st["flop"] / (te_step_ms * 1e-3) / 1e12,
                                             "workspace_bytes": te_ws_bytes},
