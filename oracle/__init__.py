@@ -14,8 +14,9 @@ Every function here follows the paper's statement of the probe:
   * head averaging, the query-frame cue A_qf, the intra-frame cue A_if and
     the cross-frame cue A_ff with its timestamp-aligned E_ff (Sec. 3.2,
     "Evidence Decomposition");
-  * the top-p block retention of the sparse prefill (Appendix, Eq. 6-9) and
-    attention restricted to the retained blocks (``topp``).
+  * the top-p block retention of the sparse prefill (Appendix, Eq. 6-9),
+    attention restricted to the retained blocks, and the coarse token-level
+    map of Eq. 10-11 with its evidence (``topp``).
 Parity pins for each function live in ``tests/test_oracle_pins.py``.
 """
 from .attention import (  # noqa: F401
@@ -24,4 +25,5 @@ from .attention import (  # noqa: F401
 )
 from .topp import (  # noqa: F401
     block_layout, block_means, select_prefix, retained_blocks, attended_mask, probe_rows_topp, evidence_topp,
+    coarse_evidence,
 )

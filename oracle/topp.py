@@ -185,3 +185,53 @@ def evidence_topp(q, k, cu_seqlens, n_vis, tokens_per_frame, block, kept, scale=
         if n_text > 0:
             aqf[fr_off[b]:fr_off[b + 1]] = frame[:, fr_off[b]:fr_off[b + 1]].sum(axis=0) / (hq * n_text)
     return tok, frame, head, aqf
+
+
+def coarse_evidence(q, k, cu_seqlens, n_vis, tokens_per_frame, block, kept, scale=None, kbar_round=None):
+    """Evidence maps from the coarse token-level map (Appendix Eq. 10-11): for a
+    text row i, a_im = q_i k_m / sqrt(d) for the keys m of its own block up to
+    i (E_i; there is no system prefix here), a_im = g_ij for the tokens of each
+    retained block K_j in S_i = ``kept[(h, row)]``, -inf elsewhere; the map is
+    the row softmax of a. Its mass on the visual tokens is summed over the
+    text rows into tok [Hq, sum n_vis], then frame, head and aqf as in the
+    exact evidence (Sec. 3.2). ``kbar_round``: see block_means."""
+    q = np.asarray(q); k = np.asarray(k)
+    n, hq, d = q.shape
+    gq = hq // k.shape[1]
+    scale = 1.0 / math.sqrt(d) if not scale else float(scale)
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    n_vis = np.asarray(n_vis, dtype=np.int64)
+    npf = int(tokens_per_frame)
+    frames = n_vis // npf
+    vis_off = np.concatenate([[0], np.cumsum(n_vis)])
+    fr_off = np.concatenate([[0], np.cumsum(frames)])
+    tok = np.zeros((hq, int(vis_off[-1])))
+    frame = np.zeros((hq, int(fr_off[-1])))
+    head = np.zeros((len(n_vis), hq))
+    aqf = np.zeros(int(fr_off[-1]))
+    for b in range(len(n_vis)):
+        s0, s1, nv = int(cu[b]), int(cu[b + 1]), int(n_vis[b])
+        n_text = s1 - s0 - nv
+        layout = block_layout(nv, n_text, block)
+        kbar = block_means(k[s0:s1], nv, n_text, block, kbar_round)
+        for h in range(hq):
+            t_map = np.zeros(nv)
+            for row in range(s0 + nv, s1):
+                pos = row - s0
+                qv = q[row, h, :].astype(np.float64)
+                a = np.full(s1 - s0, -np.inf)
+                for j in kept[(h, row)]:
+                    s, ln = layout[j]
+                    a[s:s + ln] = scale * float(kbar[j, h // gq, :] @ qv)
+                own = next(j for j, (s, ln) in enumerate(layout) if s <= pos < s + ln)
+                so, _ = layout[own]
+                a[so:pos + 1] = scale * (k[s0 + so:s0 + pos + 1, h // gq, :].astype(np.float64) @ qv)
+                w = np.exp(a - a.max())
+                t_map += (w / w.sum())[:nv]
+            tok[h, vis_off[b]:vis_off[b + 1]] = t_map
+            f_map = t_map.reshape(int(frames[b]), npf).sum(axis=1)
+            frame[h, fr_off[b]:fr_off[b + 1]] = f_map
+            head[b, h] = f_map.sum()
+        if n_text > 0:
+            aqf[fr_off[b]:fr_off[b + 1]] = frame[:, fr_off[b]:fr_off[b + 1]].sum(axis=0) / (hq * n_text)
+    return tok, frame, head, aqf

@@ -15,6 +15,7 @@ Each test names the pin it realises:
   F1-F4 the intra-frame cue A_if (closed form, dense weights, brute force, structure)
   H1-H7 top-p block retention (closed form, brute force, planted block, limits, keep-all,
         bf16 rounding of the block means, evidence with every block kept)
+  C1-C3 the coarse map of Eq. 10-11 (one-token blocks and constant keys give the exact map, mass)
   G1-G5 the cross-frame cue A_ff and E_ff (closed form, mass balance with A_if, brute force,
         dense weights, a hand-worked E_ff)
 """
@@ -739,3 +740,66 @@ def test_H7_evidence_with_every_block_kept_is_the_dense_evidence():
     want = oracle.evidence(c["q"], c["k"], c["cu"], c["n_vis"], 4)
     for g, w in zip(got, want):
         np.testing.assert_allclose(g, w, atol=1e-13)
+
+
+# Pins of oracle.topp.coarse_evidence (Appendix Eq. 10-11):
+#   C1  blocks of one token: g is the exact logit, so the coarse map is the
+#       exact attention on the same retained sets (evidence_topp)
+#   C2  constant keys: a block's mean is its keys, so again the exact map
+#   C3  mass: each text row's coarse map sums to 1, so the token map plus the
+#       rows' own-block mass is n_text per head
+def test_C1_coarse_with_one_token_blocks_is_exact():
+    c = _topp_case(51, videos=((12, 5), (8, 4)))
+    sets, _ = oracle.retained_blocks(c["q"], c["k"], c["cu"], c["n_vis"], 1, 0.8)
+    got = oracle.coarse_evidence(c["q"], c["k"], c["cu"], c["n_vis"], 4, 1, sets)
+    want = oracle.evidence_topp(c["q"], c["k"], c["cu"], c["n_vis"], 4, 1, sets)
+    for g, w in zip(got, want):
+        np.testing.assert_allclose(g, w, atol=1e-13)
+
+
+def test_C2_coarse_with_constant_keys_is_exact():
+    c = _topp_case(52, videos=((16, 6),))
+    k = np.broadcast_to(c["k"][0:1], c["k"].shape).copy()
+    sets, _ = oracle.retained_blocks(c["q"], k, c["cu"], c["n_vis"], 4, 0.7)
+    got = oracle.coarse_evidence(c["q"], k, c["cu"], c["n_vis"], 4, 4, sets)
+    want = oracle.evidence_topp(c["q"], k, c["cu"], c["n_vis"], 4, 4, sets)
+    for g, w in zip(got, want):
+        np.testing.assert_allclose(g, w, atol=1e-13)
+
+
+def test_C3_coarse_mass():
+    c = _topp_case(53, videos=((16, 6),), hq=2, hkv=1)
+    sets, _ = oracle.retained_blocks(c["q"], c["k"], c["cu"], c["n_vis"], 4, 0.9)
+    tok, frame, head, aqf = oracle.coarse_evidence(c["q"], c["k"], c["cu"], c["n_vis"], 4, 4, sets)
+    # rows 16..21 are text; their own text block (16..19 or 20..21) holds the rest of the mass
+    q, k = c["q"].astype(np.float64), c["k"].astype(np.float64)
+    for h in range(2):
+        rest = 0.0
+        for row in range(16, 22):
+            so = 16 if row < 20 else 20
+            kb = oracle.block_means(c["k"], 16, 6, 4)
+            a = {}
+            for j in sets[(h, row)]:
+                s, ln = oracle.block_layout(16, 6, 4)[j]
+                for m in range(s, s + ln):
+                    a[m] = float(kb[j, 0] @ q[row, h]) / math.sqrt(8)
+            for m in range(so, row + 1):
+                a[m] = float(k[m, 0] @ q[row, h]) / math.sqrt(8)
+            mx = max(a.values())
+            z = sum(math.exp(v - mx) for v in a.values())
+            rest += sum(math.exp(v - mx) for m, v in a.items() if m >= 16) / z
+        assert abs(tok[h].sum() + rest - 6.0) < 1e-12
+
+
+def test_C2_catches_block_sums_for_means(monkeypatch):
+    """Planted mistake: k_bar as the sum of the block's keys instead of their mean."""
+    import oracle.topp as ot
+    good = ot.block_means
+
+    def sums(k_video, n_vis, n_text, block, kbar_round=None):
+        m = good(k_video, n_vis, n_text, block, kbar_round)
+        lens = np.array([ln for _, ln in ot.block_layout(n_vis, n_text, block)], np.float64)
+        return m * lens[:, None, None]
+    monkeypatch.setattr(ot, "block_means", sums)
+    with pytest.raises(AssertionError):
+        test_C2_coarse_with_constant_keys_is_exact()
