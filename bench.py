@@ -473,6 +473,15 @@ def bench_ours(args, cfg):
 
     tpp_ms = _time(probe_topp)
     tp_tiles = int(tp_row_ptr[-1])
+    # the evidence of the coarse token-level map (Eq. 10-11) on the same sets
+    ev.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, npf, 0.97, ws=ws_tp)
+    maps_co = [torch.empty_like(m) for m in maps]
+
+    def coarse():
+        ev.evisel_coarse_evidence(q, k, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, npf, keep_tp, ws_tp,
+                                  tok=maps_co[0], frame=maps_co[1], head=maps_co[2], aqf=maps_co[3])
+
+    co_ms = _time(coarse)
     status = ev.evisel_status(ws_tp)
     ws_tp.free()
     del keep_tp, uni_tp
@@ -513,7 +522,7 @@ def bench_ours(args, cfg):
                                 "tflops": if_flop / (if_ms * 1e-3) / 1e12},
                 "topp_mask": {"ms": tp_ms, "block": npf, "tau_p": 0.97, "blocks": n_blk,
                               "tflops_history": tp_flop / (tp_ms * 1e-3) / 1e12,
-                              "probe_ms": tpp_ms, "union_tiles": tp_tiles,
+                              "probe_ms": tpp_ms, "union_tiles": tp_tiles, "coarse_evidence_ms": co_ms,
                               "static_mask_tiles": int(probe.row_ptr[-1])},
                 "text_evidence_recompute": {"step_ms": te_step_ms, "probe_ms": te_probe_ms, "evidence_ms": te_ev_ms,
                                             "tflops": st["flop"] / (te_step_ms * 1e-3) / 1e12,

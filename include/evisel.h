@@ -280,6 +280,27 @@ int evisel_topp_mask(const evisel_probe_args* args, int32_t block, float tau_p, 
                      uint32_t* tile_union, void* stream, evisel_ws** ws_inout);
 
 /* ---------------------------------------------------------------------------
+ * evisel_coarse_evidence: the evidence maps of the coarse token-level map of the
+ * sparse prefill (Appendix, "Detailed Sparse Prefilling", Eq. 10-11). For a text
+ * row i of head h: a_im = softmax_scale q_i k_m for the keys of its own block up
+ * to i, a_im = g_ij = softmax_scale q_i k_bar_j for the tokens of each block j of
+ * S_i, -inf elsewhere; A~_i = softmax(a_i). Then, over the text rows,
+ *   tok[h, m] = sum_i A~_im (visual m), frame[h, t], head[b, h], aqf[t]
+ * as evisel_evidence_reduce() defines them (same layouts).
+ *   args   as for the evisel_topp_mask() call that ran on `ws` (q, k, videos, N_v,
+ *          heads, head_dim, softmax_scale); `block` its block size.
+ *   keep   that call's per-row bits (S_i and the own block).
+ *   ws     the workspace of that call (its k_bar is read; coarse scratch grows
+ *          by about hq * n_text_total * 32 * W * 4 bytes).
+ *   accumulate  0: overwrite tok and frame; 1: add (sum over layers); head and
+ *          aqf are recomputed from the resulting frame map.
+ * Asynchronous on `stream` after a short synchronous upload of the per-video
+ * offsets. Errors: EVISEL_EINVAL, EVISEL_ESTATE (no evisel_topp_mask on ws),
+ * EVISEL_ENOMEM, EVISEL_ECUDA. */
+int evisel_coarse_evidence(const evisel_probe_args* args, evisel_ws* ws, int32_t block, const uint32_t* keep,
+                           float* tok, float* frame, float* head, float* aqf, int accumulate, void* stream);
+
+/* ---------------------------------------------------------------------------
  * evisel_selftest_wait: failure detection check (no counterpart in the paper).
  * Every wait in the library's kernels is bounded: it gives up after a time
  * limit, records EVISEL_ETIMEOUT in a device status word and lets the kernel

@@ -7,6 +7,7 @@ the same entry-point names. ``workloads`` draws the seeded synthetic inputs.
 from ._binding import (  # noqa: F401
     EviselError, Workspace, evisel_evidence_reduce, evisel_free, evisel_probe_attention, evisel_probe_evidence_noalloc,
     evisel_intra_frame_evidence, evisel_cross_frame_evidence, evisel_topp_mask, tile_union_to_csr,
+    evisel_coarse_evidence,
     evisel_selftest_wait, evisel_status, load,
 )
 

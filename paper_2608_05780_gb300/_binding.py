@@ -90,6 +90,8 @@ def load(path: str = LIB_PATH):
     lib.evisel_cross_frame_evidence.restype = i32
     lib.evisel_topp_mask.argtypes = [ctypes.POINTER(ProbeArgs), i32, ctypes.c_float, vp, vp, vp, ctypes.POINTER(vp)]
     lib.evisel_topp_mask.restype = i32
+    lib.evisel_coarse_evidence.argtypes = [ctypes.POINTER(ProbeArgs), vp, i32, vp, vp, vp, vp, vp, i32, vp]
+    lib.evisel_coarse_evidence.restype = i32
     lib.evisel_selftest_wait.argtypes = [i32, i32, vp, ctypes.POINTER(ctypes.c_int)]
     lib.evisel_selftest_wait.restype = i32
     _lib = lib
@@ -354,3 +356,32 @@ def tile_union_to_csr(tile_union, n_vis, tile):
             row_ptr.append(len(cols))
             r += 1
     return np.array(row_ptr, np.int32), np.array(cols, np.int32)
+
+
+def evisel_coarse_evidence(q, k, cu_seqlens, n_vis, tokens_per_frame, tile, block, keep, ws, tok=None, frame=None,
+                           head=None, aqf=None, accumulate=False, softmax_scale=0.0, stream=None):
+    """Evidence maps of the coarse token-level map (Appendix Eq. 10-11) on the
+    evisel_topp_mask call that ran on ``ws`` (``keep`` its bits).
+
+    Returns (tok [hq, sum n_vis], frame [hq, sum T], head [B, hq], aqf [sum T])."""
+    import torch
+    lib = load()
+    nv = np.asarray(n_vis, dtype=np.int64)
+    hq = int(q.shape[1])
+    total_vis = int(nv.sum())
+    frames = int((nv // int(tokens_per_frame)).sum())
+    dev = q.device
+    tok = torch.empty((hq, total_vis), device=dev) if tok is None else tok
+    frame = torch.empty((hq, frames), device=dev) if frame is None else frame
+    head = torch.empty((len(nv), hq), device=dev) if head is None else head
+    aqf = torch.empty((frames,), device=dev) if aqf is None else aqf
+    dummy = torch.empty(0, device=dev)
+    args, keepalive = make_args(q, k, k, cu_seqlens, n_vis, tokens_per_frame, tile, [0], [], dummy, dummy,
+                                softmax_scale)
+    _check(lib.evisel_coarse_evidence(ctypes.byref(args), ws.ptr, int(block), keep.data_ptr(),
+                                      tok.data_ptr() if tok.numel() else None,
+                                      frame.data_ptr() if frame.numel() else None, head.data_ptr(),
+                                      aqf.data_ptr() if aqf.numel() else None, int(bool(accumulate)),
+                                      _stream_handle(stream)))
+    del keepalive
+    return tok, frame, head, aqf

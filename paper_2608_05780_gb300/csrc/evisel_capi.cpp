@@ -388,6 +388,12 @@ struct evisel_ws {
   void* topp_stage = nullptr;
   size_t topp_stage_bytes = 0;
   cudaEvent_t topp_done = nullptr;
+  int topp_block = 0;               // the last evisel_topp_mask on this workspace
+  int topp_n_videos = 0, topp_n_words = 0, topp_n_tok = 0;
+  size_t topp_kbar_off = 0;
+  // coarse map scratch: offsets, block affinities and row normalisers of the text rows
+  void* coarse_buf = nullptr;
+  size_t coarse_bytes = 0;
 };
 
 namespace {
@@ -904,6 +910,96 @@ int evisel_topp_mask(const evisel_probe_args* a, int32_t block, float tau_p, uin
   e = launch_topp(L, stream);
   if (e != cudaSuccess) return cuda_fail(e, "top-p launch");
   ws->last_stream = stream;
+  ws->topp_block = block;
+  ws->topp_n_videos = a->num_videos;
+  ws->topp_n_words = n_words;
+  ws->topp_n_tok = n_tok;
+  ws->topp_kbar_off = meta;
+  return EVISEL_OK;
+}
+
+int evisel_coarse_evidence(const evisel_probe_args* a, evisel_ws* ws, int32_t block, const uint32_t* keep, float* tok,
+                           float* frame, float* head, float* aqf, int accumulate, void* stream_ptr) {
+  g_last_error.clear();
+  if (!a || !ws) return fail(EVISEL_EINVAL, "args or workspace is NULL");
+  if (ws->topp_block == 0) return fail(EVISEL_ESTATE, "no evisel_topp_mask has run on this workspace");
+  if (block != ws->topp_block || a->num_videos != ws->topp_n_videos ||
+      (a->num_videos > 0 && a->cu_seqlens_h[a->num_videos] != ws->topp_n_tok))
+    return fail(EVISEL_EINVAL, "args / block do not match the evisel_topp_mask call on this workspace");
+  if (a->num_videos == 0) return EVISEL_OK;
+  const int npf = a->tokens_per_frame;
+  std::vector<int> text_off(1, 0), vis_off(1, 0), frame_off(1, 0);
+  int max_frames = 0;
+  for (int b = 0; b < a->num_videos; ++b) {
+    const int nv = a->n_vis_h[b], nt = a->cu_seqlens_h[b + 1] - a->cu_seqlens_h[b] - nv;
+    text_off.push_back(text_off.back() + nt);
+    vis_off.push_back(vis_off.back() + nv);
+    frame_off.push_back(frame_off.back() + nv / npf);
+    max_frames = std::max(max_frames, nv / npf);
+  }
+  const int total_text = text_off.back();
+  if ((vis_off.back() > 0 && (!tok || !frame)) || !head || (frame_off.back() > 0 && !aqf) || !keep || !a->q || !a->k)
+    return fail(EVISEL_EINVAL, "an output map, keep, q or k is NULL");
+  const int pitch = ws->topp_n_words * 32;
+  const size_t ints = align_up(3 * (a->num_videos + 1) * sizeof(int), 256);
+  const size_t gbytes = align_up(static_cast<size_t>(a->hq) * total_text * pitch * sizeof(float), 256);
+  const size_t mz = align_up(static_cast<size_t>(a->hq) * total_text * sizeof(float), 256);
+  const size_t need = ints + gbytes + 2 * mz;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_ptr);
+  if (need > ws->coarse_bytes) {
+    cudaStreamSynchronize(ws->last_stream);
+    cudaStreamSynchronize(stream);
+    if (ws->coarse_buf) cudaFree(ws->coarse_buf);
+    ws->coarse_buf = nullptr;
+    ws->coarse_bytes = 0;
+    if (cudaMalloc(&ws->coarse_buf, need) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(EVISEL_ENOMEM, "coarse-map scratch of " + std::to_string(need) + " bytes");
+    }
+    ws->coarse_bytes = need;
+  }
+  std::vector<int> offs;
+  offs.insert(offs.end(), text_off.begin(), text_off.end());
+  offs.insert(offs.end(), vis_off.begin(), vis_off.end());
+  offs.insert(offs.end(), frame_off.begin(), frame_off.end());
+  char* d = static_cast<char*>(ws->coarse_buf);
+  cudaError_t e = cudaMemcpyAsync(d, offs.data(), offs.size() * sizeof(int), cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);   // the host vector goes out of scope
+  if (e != cudaSuccess) return cuda_fail(e, "coarse-map offsets");
+  CoarseLaunch L{};
+  L.q = a->q;
+  L.k = a->k;
+  L.kbar = static_cast<char*>(ws->topp_buf) + ws->topp_kbar_off;
+  L.vids = static_cast<const ToppVideo*>(ws->topp_buf);
+  L.text_off = reinterpret_cast<const int*>(d);
+  L.vis_off = L.text_off + (a->num_videos + 1);
+  L.frame_off = L.vis_off + (a->num_videos + 1);
+  L.keep = keep;
+  L.gbuf = reinterpret_cast<float*>(d + ints);
+  L.row_m = reinterpret_cast<float*>(d + ints + gbytes);
+  L.row_z = reinterpret_cast<float*>(d + ints + gbytes + mz);
+  L.tok = tok;
+  L.frame = frame;
+  L.head = head;
+  L.aqf = aqf;
+  L.n_videos = a->num_videos;
+  L.total_text = total_text;
+  L.pitch = pitch;
+  L.n_words = ws->topp_n_words;
+  L.n_tok = ws->topp_n_tok;
+  L.hq = a->hq;
+  L.hkv = a->hkv;
+  L.head_dim = a->head_dim;
+  L.block = block;
+  L.tokens_per_frame = npf;
+  L.total_vis = vis_off.back();
+  L.total_frames = frame_off.back();
+  L.max_frames = max_frames;
+  L.accumulate = accumulate != 0;
+  L.scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / std::sqrt(float(a->head_dim));
+  e = launch_coarse(L, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "coarse-map launch");
+  ws->last_stream = stream;
   return EVISEL_OK;
 }
 
@@ -920,6 +1016,7 @@ void evisel_free(evisel_ws* ws) {
   if (ws->stage_done) cudaEventDestroy(ws->stage_done);
   if (ws->topp_done) cudaEventSynchronize(ws->topp_done);
   if (ws->topp_buf) cudaFree(ws->topp_buf);
+  if (ws->coarse_buf) cudaFree(ws->coarse_buf);
   if (ws->topp_stage) cudaFreeHost(ws->topp_stage);
   if (ws->topp_done) cudaEventDestroy(ws->topp_done);
   if (prev >= 0 && prev != ws->device) cudaSetDevice(prev);

@@ -222,6 +222,30 @@ struct ToppLaunch {
 cudaError_t launch_intra_frame(const IntraFrameLaunch& L, cudaStream_t stream);
 cudaError_t launch_text_evidence(const TextEvidenceLaunch& L, cudaStream_t stream);
 cudaError_t launch_topp(const ToppLaunch& L, cudaStream_t stream);
+
+// Evidence from the coarse token-level map (Eq. 10-11), on the builder's k_bar and keep bits.
+struct CoarseLaunch {
+  const void* q;                    // bf16 [N, hq, d]
+  const void* k;                    // bf16 [N, hkv, d]
+  const void* kbar;                 // bf16 [blocks, hkv, d] (from the builder)
+  const ToppVideo* vids;
+  const int* text_off;              // [videos + 1] first text row of each video (text rows back to back)
+  const int* vis_off;               // [videos + 1] column offsets of the token map
+  const int* frame_off;             // [videos + 1] column offsets of the frame map
+  const uint32_t* keep;             // [hq, n_words, N]
+  float* gbuf;                      // [hq, total_text, pitch] block affinities of the text rows
+  float* row_m;                     // [hq, total_text]
+  float* row_z;                     // [hq, total_text]
+  float* tok;
+  float* frame;
+  float* head;
+  float* aqf;
+  int n_videos, total_text, pitch, n_words, n_tok, hq, hkv, head_dim, block, tokens_per_frame;
+  int total_vis, total_frames, max_frames, accumulate;
+  float scale;
+};
+
+cudaError_t launch_coarse(const CoarseLaunch& L, cudaStream_t stream);
 cudaError_t launch_cross_frame(const CrossFrameLaunch& L, cudaStream_t stream);
 cudaError_t launch_probe_attn(const ProbeLaunch& L, cudaStream_t stream);
 cudaError_t launch_attn_combine(const CombineLaunch& L, cudaStream_t stream);

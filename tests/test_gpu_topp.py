@@ -210,3 +210,33 @@ def test_keep_refused_where_it_does_not_apply(cuda_lib):
                                              row_ptr, col_idx, o, lse, ws)
     torch.cuda.synchronize()
     ws.free()
+
+
+@pytest.mark.parametrize("name,block,tau", [("single", 16, 0.5), ("tiny", 16, 0.9)])
+def test_coarse_evidence_matches_oracle(cuda_lib, name, block, tau):
+    """Evidence of the coarse map (Eq. 10-11) on the GPU's own retained sets
+    against the oracle taken with the same sets and bf16 block means."""
+    import torch
+    from gpu_helpers import check_maps, np32
+    probe = wl.make_probe(wl.CONFIGS[name])
+    cfg = probe.cfg
+    q, k, v = to_device(probe)
+    keep, uni, ws = cuda_lib.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                              block, tau)
+    maps = cuda_lib.evisel_coarse_evidence(q, k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                           block, keep, ws)
+    torch.cuda.synchronize()
+    assert cuda_lib.evisel_status(ws) == 0
+    n = int(probe.cu_seqlens[-1])
+    text_rows = np.concatenate([np.arange(int(probe.cu_seqlens[b]) + int(probe.n_vis[b]), int(probe.cu_seqlens[b + 1]))
+                                for b in range(len(probe.n_vis))])
+    kept = _sets_from_keep(keep, text_rows, probe.cu_seqlens, probe.n_vis, block)
+    want = oracle.coarse_evidence(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, block, kept,
+                                  kbar_round="bf16")
+    check_maps([np32(m) for m in maps], list(want), probe, label=f"{name} coarse evidence")
+    # accumulate: a second call adds the same maps
+    maps2 = cuda_lib.evisel_coarse_evidence(q, k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                            block, keep, ws, tok=maps[0].clone(), frame=maps[1].clone(),
+                                            head=maps[2].clone(), aqf=maps[3].clone(), accumulate=True)
+    check_maps([np32(m) for m in maps2], [2 * w for w in want], probe, layers=2, label=f"{name} coarse x2")
+    ws.free()
