@@ -488,8 +488,8 @@ def bench_ours(args, cfg):
     if status != 0:
         raise RuntimeError("device status reported an error")
     n_blk = int(sum(int(nv) // npf + -(-int(nt) // npf) for nv, nt in zip(probe.n_vis, probe.n_text)))
-    # algorithmic tensor work: 4 passes of q k_bar^T over each row's history, head by head
-    tp_flop = 4 * 2.0 * d * hq * sum(
+    # tensor work of the builder: 6 passes of q k_bar^T over each row's history, head by head
+    tp_flop = 6 * 2.0 * d * hq * sum(
         sum((p_ // npf) for p_ in range(int(nv))) + sum(int(nv) // npf + t // npf for t in range(int(nt)))
         for nv, nt in zip(probe.n_vis, probe.n_text))
     te_probe_ms = _time(probe_te)

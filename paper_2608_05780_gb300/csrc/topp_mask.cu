@@ -14,15 +14,19 @@
 // topp_select_kernel: one CTA per (128-row tile of a video, KV group), 192
 //   threads (warp 4 TMA, warp 5 MMA, warps 0-3 one row each). For each head of
 //   the group, S = Q_h k_bar^T in chunks of 128 blocks (tcgen05, TMEM double
-//   buffer), in four passes over the chunks:
-//     0  the row's max and min logit over H_i and the softmax sum Z (online);
-//     1  the mass per bin of 128 equal logit bins between max and min; the
-//        bin b1 where the cumulative mass from the top reaches tau_p Z;
-//     2  the same with 128 sub-bins of bin b1: sub-bin b2;
-//     3  keep every block of a higher bin or sub-bin; inside sub-bin b2,
-//        blocks in id order while the mass before them is below tau_p Z.
-//   The blocks are ordered by logit as exactly as the sub-bin width
-//   ((max - min) / 16384) resolves them; closer logits count as ties.
+//   buffer), in six passes over the chunks:
+//     0     the row's max and min logit over H_i and the softmax sum Z (online);
+//     1..4  a radix select on the block's key q = floor((max - x) 2^14 / (max -
+//           min)) (0 = the largest logit), digit by digit (3, 3, 4 and 4 bits,
+//           top first): the mass per digit value of the blocks whose higher
+//           digits equal the boundary's, in 8 or 16 register bins; the boundary
+//           digit is the one where the cumulative mass from the top reaches
+//           tau_p Z;
+//     5     keep every block whose key is below the boundary key; at the
+//           boundary key, blocks in id order while the mass before them is
+//           below tau_p Z.
+//   The blocks are ordered by logit as exactly as the key resolves them
+//   ((max - min) / 16384); closer logits count as ties.
 // topp_union_kernel: one thread per (row, head) ORs its bits, mapped to key
 //   tiles, into its attention row tile's union.
 // Every wait is bounded; a timeout records EVISEL_ETIMEOUT.
@@ -38,11 +42,14 @@ namespace {
 
 constexpr int kRows = 128;
 constexpr int kCols = 128;                       // blocks per chunk
-constexpr int kBins = 128;
 constexpr int kThreads = 192;
 constexpr int kWarpProducer = 4;
 constexpr int kWarpMma = 5;
-constexpr int kPasses = 4;
+constexpr int kQBits = 14;                       // key resolution: (max - min) / 2^14 over H_i
+constexpr int kQMax = (1 << kQBits) - 1;
+constexpr int kLevels = 4;                       // key digits of 3, 3, 4 and 4 bits
+constexpr int kDigBins = 16;
+constexpr int kPasses = kLevels + 2;             // stats, one pass per digit, bits
 
 template <int D>
 struct TpCfg {
@@ -51,8 +58,8 @@ struct TpCfg {
   static constexpr int BLOCK = kRows * 128;
   static constexpr int OFF_Q = 0;                     // 2 stages (one per head in flight)
   static constexpr int OFF_K = 2 * TILE_BYTES;        // 2 stages of k_bar chunks
-  static constexpr int OFF_HIST = OFF_K + 2 * TILE_BYTES;   // [kBins][128] fp32
-  static constexpr int OFF_BAR = OFF_HIST + kBins * kRows * 4;
+  static constexpr int OFF_STASH = OFF_K + 2 * TILE_BYTES;   // [32][128] fp32: a group's u, per row
+  static constexpr int OFF_BAR = OFF_STASH + 32 * kRows * 4;
   static constexpr int B_QF = 0, B_QE = 2, B_KF = 4, B_KE = 6, B_SF = 8, B_SE = 10, B_DRAIN = 12;
   static constexpr int N_BARS = 13;
   static constexpr int OFF_MISC = OFF_BAR + N_BARS * 8;
@@ -60,6 +67,24 @@ struct TpCfg {
   static constexpr int TMEM_COLS = 256;
   static_assert(SMEM_BYTES <= 232448, "shared memory budget");
 };
+
+// acc[K] += w for K = d, K < N (no bin for other d): a predicated add per
+// bin with static register indices.
+template <int K, int N>
+__device__ __forceinline__ void bin_add(float (&acc)[kDigBins], int d, float w) {
+  if constexpr (K < N) {
+    asm("{\n\t.reg .pred p;\n\tsetp.eq.s32 p, %1, %2;\n\t@p add.rn.f32 %0, %0, %3;\n\t}"
+        : "+f"(acc[K]) : "r"(d), "n"(K), "f"(w));
+    bin_add<K + 1, N>(acc, d, w);
+  }
+}
+
+// Digit lv of the key (top first): width and shift.
+__host__ __device__ constexpr int digit_width(int lv) { return lv < 2 ? 3 : 4; }
+__host__ __device__ constexpr int digit_shift(int lv) {
+  return lv == 0 ? kQBits - 3 : lv == 1 ? kQBits - 6 : lv == 2 ? kQBits - 10 : 0;
+}
+static_assert(digit_shift(kLevels - 1) == 0 && digit_shift(2) == digit_width(3), "digits cover the key");
 
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
   const bool ok = ptx::mbar_wait(bar, parity, abort_flag, kWaitTimeoutNs);
@@ -113,7 +138,7 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
   };
   const int nh_max = n_hist(rt.local0 + rt.q_len - 1);
   const int n_ch = (nh_max + kCols - 1) / kCols;
-  const int n_steps = gq * kPasses * n_ch;       // step t: head t / (4 n_ch), pass (t / n_ch) % 4, chunk t % n_ch
+  const int n_steps = gq * kPasses * n_ch;       // step t: head t / (kPasses n_ch), pass (t / n_ch) % kPasses, chunk t % n_ch
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < C::N_BARS; ++i) ptx::mbar_init(bar(i), (i == C::B_SE || i == C::B_SE + 1) ? kRows : 1u);
@@ -229,27 +254,35 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
     const int pos = rt.local0 + row;
     const int nh = row_ok ? n_hist(pos) : 0;
     const uint32_t tbase = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    float* hist = reinterpret_cast<float*>(smem + C::OFF_HIST) + row;   // column of this thread: hist[bin * 128]
     const float sc = L.scale_log2;               // logits in log2 units
+    float* stash = reinterpret_cast<float*>(smem + C::OFF_STASH) + row;   // this row's column: stash[e * 128]
     bool ok = true;
     for (int hh = 0; hh < gq; ++hh) {
       const int h = g * gq + hh;
       float m = -INFINITY, gmin = INFINITY, z = 0.f;
-      float w1 = 0.f, inv_w1 = 0.f, inv_w2 = 0.f, target = 0.f, above1 = 0.f, above2 = 0.f, tie = 0.f;
-      int b1 = 0, b2 = 0;
+      float inv_r = 0.f, target = 0.f, above = 0.f, tie = 0.f;
+      int wkey = 0;                              // the boundary's key digits found so far
       uint32_t* keep = L.keep + static_cast<int64_t>(h) * L.n_words * L.n_tok + rt.q_start + row;
       for (int pass = 0; pass < kPasses; ++pass) {
-        if (pass == 1 || pass == 2) {
-          for (int bi = 0; bi < kBins; ++bi) hist[bi * kRows] = 0.f;
-        }
+        const int lv = pass - 1;                 // digit of passes 1..kLevels
+        const int width = digit_width(lv), dshift = digit_shift(lv);
+        const int pshift = dshift + width;       // key >> pshift: the digits above this one
+        // The window (keys with the boundary's higher digits) as bounds on v =
+        // (max - x) 2^14 / (max - min): key = min(kQMax, floor(v)), so
+        // key >> pshift == wkey iff lo <= v < hi (hi open at the top key).
+        const float lo = static_cast<float>(wkey << pshift);
+        const float hi = ((wkey + 1) << pshift) > kQMax ? INFINITY : static_cast<float>((wkey + 1) << pshift);
+        float acc[kDigBins];
+#pragma unroll
+        for (int k = 0; k < kDigBins; ++k) acc[k] = 0.f;
         for (int ch = 0; ch < n_ch; ++ch) {
           const int t = (hh * kPasses + pass) * n_ch + ch, b = t % 2;
           ok = ok && warp_wait(bar(C::B_SF + b), (t / 2) & 1, abort_flag);
-          int run_bin = -1;                        // histogram passes: consecutive keys of one bin add in a register
-          float run = 0.f;
           if (ok && __any_sync(0xffffffffu, nh > ch * kCols)) {   // warp-uniform: tcgen05.ld is collective
             ptx::tc_fence_after();
-            // One compact loop per pass (uniform over the warp), 32 columns at a time.
+            // One compact loop per pass (uniform over the warp), 32 columns at a
+            // time. x, the key and the weight use non-contracted arithmetic so
+            // that every pass sees the same values.
 #pragma unroll 1
             for (int c0 = 0; c0 < kCols; c0 += 32) {
               uint32_t r[32];
@@ -257,71 +290,83 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
               ptx::tmem_wait_ld();
               const int jn = nh - (ch * kCols + c0);         // columns e < jn are in H_i
               if (pass == 0) {
-                float cmax = -INFINITY;
+                float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                float mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                  const float x = __uint_as_float(r[e]) * sc;
+                  const float x = __fmul_rn(__uint_as_float(r[e]), sc);
                   if (e < jn) {
-                    cmax = fmaxf(cmax, x);
-                    gmin = fminf(gmin, x);
+                    mx[e & 3] = fmaxf(mx[e & 3], x);
+                    mn[e & 3] = fminf(mn[e & 3], x);
                   }
                 }
+                const float cmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+                gmin = fminf(gmin, fminf(fminf(mn[0], mn[1]), fminf(mn[2], mn[3])));
                 if (cmax > m) {
                   z = (m == -INFINITY) ? 0.f : z * ptx::ex2(m - cmax);
                   m = cmax;
                 }
-                float zs = 0.f;
+                float zs[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                 for (int e = 0; e < 32; ++e)
-                  if (e < jn) zs += ptx::ex2(__uint_as_float(r[e]) * sc - m);
-                z += zs;
-              } else if (pass == 1) {
+                  if (e < jn) zs[e & 3] += ptx::ex2(__fsub_rn(__fmul_rn(__uint_as_float(r[e]), sc), m));
+                z += (zs[0] + zs[1]) + (zs[2] + zs[3]);
+              } else if (lv == 0) {
+                // The first digit (every column is in the window): no branches,
+                // so that the columns' arithmetic overlaps.
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                  if (e >= jn) break;
-                  const float x = __uint_as_float(r[e]) * sc;
-                  const int bin1 = min(kBins - 1, static_cast<int>((m - x) * inv_w1));
-                  if (bin1 != run_bin) {
-                    if (run_bin >= 0) hist[run_bin * kRows] += run;
-                    run_bin = bin1;
-                    run = 0.f;
-                  }
-                  run += ptx::ex2(x - m);
+                  const float u = __fsub_rn(m, __fmul_rn(__uint_as_float(r[e]), sc));
+                  const float v = __fmul_rn(u, inv_r);
+                  const int key = min(kQMax, __float2int_rz(v));
+                  const int dig = (e < jn && v >= lo && v < hi) ? (key >> dshift) & ((1 << width) - 1) : -1;
+                  bin_add<0, 8>(acc, dig, ptx::ex2(-u));
                 }
-              } else if (pass == 2) {
+              } else if (lv < kLevels) {
+                // Later digits (a few percent of the columns): the window test stashes the
+                // window's u; then each lane walks its own window columns in id
+                // order and adds ex2(-u) to the digit's bin.
+                uint32_t in_mask = 0u;
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                  if (e >= jn) break;
-                  const float x = __uint_as_float(r[e]) * sc;
-                  const float u = m - x;
-                  if (min(kBins - 1, static_cast<int>(u * inv_w1)) != b1) continue;
-                  const int bin2 = min(kBins - 1, static_cast<int>((u - b1 * w1) * inv_w2));
-                  if (bin2 != run_bin) {
-                    if (run_bin >= 0) hist[run_bin * kRows] += run;
-                    run_bin = bin2;
-                    run = 0.f;
+                  const float u = __fsub_rn(m, __fmul_rn(__uint_as_float(r[e]), sc));
+                  const float v = __fmul_rn(u, inv_r);
+                  if (e < jn && v >= lo && v < hi) {
+                    in_mask |= 1u << e;
+                    stash[e * kRows] = u;
                   }
-                  run += ptx::ex2(x - m);
                 }
+                while (in_mask != 0u) {
+                  const int e = __ffs(in_mask) - 1;
+                  in_mask &= in_mask - 1u;
+                  const float u = stash[e * kRows];
+                  const int key = min(kQMax, __float2int_rz(__fmul_rn(u, inv_r)));
+                  bin_add<0, 16>(acc, (key >> dshift) & ((1 << width) - 1), ptx::ex2(-u));
+                }
+                __syncwarp();
               } else {
-                uint32_t word = 0u;
+                // key < wkey iff v < wkey; key == wkey iff wkey <= v < wkey + 1 (open at the top key)
+                const float k0 = static_cast<float>(wkey);
+                const float k1 = wkey == kQMax ? INFINITY : static_cast<float>(wkey + 1);
+                uint32_t word = 0u, at_mask = 0u;
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                  if (e >= jn) break;
-                  const float x = __uint_as_float(r[e]) * sc;
-                  const float u = m - x;
-                  const int bin1 = min(kBins - 1, static_cast<int>(u * inv_w1));
-                  bool kept = bin1 < b1;
-                  if (bin1 == b1) {
-                    const int bin2 = min(kBins - 1, static_cast<int>((u - b1 * w1) * inv_w2));
-                    kept = bin2 < b2;
-                    if (bin2 == b2) {                             // ties: lower ids first
-                      kept = above2 + tie < target;
-                      tie += ptx::ex2(x - m);
-                    }
+                  const float u = __fsub_rn(m, __fmul_rn(__uint_as_float(r[e]), sc));
+                  const float v = __fmul_rn(u, inv_r);
+                  word |= (e < jn && v < k0) ? 1u << e : 0u;
+                  if (e < jn && v >= k0 && v < k1) {
+                    at_mask |= 1u << e;
+                    stash[e * kRows] = u;
                   }
-                  if (kept) word |= 1u << e;
                 }
+                // the boundary key: lower ids first while the mass before them is below the target
+                while (at_mask != 0u) {
+                  const int e = __ffs(at_mask) - 1;
+                  at_mask &= at_mask - 1u;
+                  if (above + tie < target) word |= 1u << e;
+                  tie += ptx::ex2(-stash[e * kRows]);
+                }
+                __syncwarp();
                 const int w = ch * 4 + (c0 >> 5);
                 if (row_ok && w < L.n_words) {
                   if (w == nh >> 5) word |= 1u << (nh & 31);     // the row's own block
@@ -330,7 +375,7 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
               }
             }
             ptx::tc_fence_before();
-          } else if (pass == 3 && row_ok && ok) {
+          } else if (pass == kPasses - 1 && row_ok && ok) {
             // No column of this chunk is in H_i for the warp: zeros (and the own block).
             for (int wi = 0; wi < 4; ++wi) {
               const int w = ch * 4 + wi;
@@ -339,41 +384,32 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
             }
           }
           ptx::mbar_arrive(bar(C::B_SE + b));
-          if (run_bin >= 0) hist[run_bin * kRows] += run;
         }
-        // Between passes: the bin widths and the boundary (bin, mass above it).
-        // A boundary is the first bin whose cumulative mass from the top reaches
-        // the target; when rounding keeps the total below it (tau_p near 1), the
-        // last non-empty bin, whose members are then all kept.
+        // Between passes: the key scale, then per digit the boundary value and
+        // the mass above it. The boundary is the first digit value whose
+        // cumulative mass from the top reaches the target; when rounding keeps
+        // the total below it (tau_p near 1), the last non-empty one, whose
+        // blocks are then all kept.
         if (pass == 0) {
           target = L.tau * z;
-          w1 = fmaxf((m - gmin) / kBins, 1e-30f);
-          inv_w1 = 1.f / w1;
-          inv_w2 = static_cast<float>(kBins) * inv_w1;
-        } else if (pass == 1 || pass == 2) {
-          float acc = pass == 1 ? 0.f : above1, before_last = acc;
+          inv_r = static_cast<float>(kQMax + 1) / fmaxf(m - gmin, 1e-30f);
+        } else if (lv < kLevels) {
+          float run = above, before_last = above;
           int found = -1, last = 0;
-          for (int bi = 0; bi < kBins; ++bi) {
-            const float hb = hist[bi * kRows];
+#pragma unroll
+          for (int k = 0; k < kDigBins; ++k) {
+            const float hb = acc[k];
             if (hb > 0.f) {
-              last = bi;
-              before_last = acc;
+              last = k;
+              before_last = run;
             }
-            if (acc + hb >= target) {
-              found = bi;
-              break;
+            if (found < 0) {
+              if (run + hb >= target) found = k;
+              else run += hb;
             }
-            acc += hb;
           }
-          const int bb = found >= 0 ? found : last;
-          const float ab = found >= 0 ? acc : before_last;
-          if (pass == 1) {
-            b1 = bb;
-            above1 = ab;
-          } else {
-            b2 = bb;
-            above2 = ab;
-          }
+          above = found >= 0 ? run : before_last;
+          wkey = (wkey << width) | (found >= 0 ? found : last);
         }
       }
       // The own block's word when it lies past the chunks of this tile.
