@@ -11,10 +11,11 @@
 //
 // kbar_kernel: one CTA per (block, KV head): the block's mean key in fp32,
 //   stored as bf16 (the tensor cores' input type).
-// topp_select_kernel: one CTA per (128-row tile of a video, KV group), 192
-//   threads (warp 4 TMA, warp 5 MMA, warps 0-3 one row each). For each head of
-//   the group, S = Q_h k_bar^T in chunks of 128 blocks (tcgen05, TMEM double
-//   buffer), in six passes over the chunks:
+// topp_select_kernel: one CTA per (128-row tile of a video, KV group), 320
+//   threads (warp 8 TMA, warp 9 MMA; warps 0-7 one row each, of head slot
+//   warp / 4). The heads of the group go in pairs: S = Q_h k_bar^T for both
+//   heads of a pair, in chunks of 128 blocks (tcgen05, both products from one
+//   k_bar chunk, TMEM 2 buffers x 2 heads), in six passes over the chunks:
 //     0     the row's max and min logit over H_i and the softmax sum Z (online);
 //     1..4  a radix select on the block's key q = floor((max - x) 2^14 / (max -
 //           min)) (0 = the largest logit), digit by digit (3, 3, 4 and 4 bits,
@@ -42,9 +43,11 @@ namespace {
 
 constexpr int kRows = 128;
 constexpr int kCols = 128;                       // blocks per chunk
-constexpr int kThreads = 192;
-constexpr int kWarpProducer = 4;
-constexpr int kWarpMma = 5;
+constexpr int kHeadSlots = 2;                    // heads in flight
+constexpr int kRowWarps = 4 * kHeadSlots;        // warp w: rows 32 (w % 4) .. of head slot w / 4
+constexpr int kWarpProducer = kRowWarps;
+constexpr int kWarpMma = kRowWarps + 1;
+constexpr int kThreads = 32 * (kRowWarps + 2);
 constexpr int kQBits = 14;                       // key resolution: (max - min) / 2^14 over H_i
 constexpr int kQMax = (1 << kQBits) - 1;
 constexpr int kLevels = 4;                       // key digits of 3, 3, 4 and 4 bits
@@ -56,15 +59,15 @@ struct TpCfg {
   static constexpr int KB = D / 64;
   static constexpr int TILE_BYTES = kRows * D * 2;   // 128 rows (Q) or 128 blocks (k_bar)
   static constexpr int BLOCK = kRows * 128;
-  static constexpr int OFF_Q = 0;                     // 2 stages (one per head in flight)
-  static constexpr int OFF_K = 2 * TILE_BYTES;        // 2 stages of k_bar chunks
-  static constexpr int OFF_STASH = OFF_K + 2 * TILE_BYTES;   // [32][128] fp32: a group's u, per row
-  static constexpr int OFF_BAR = OFF_STASH + 32 * kRows * 4;
-  static constexpr int B_QF = 0, B_QE = 2, B_KF = 4, B_KE = 6, B_SF = 8, B_SE = 10, B_DRAIN = 12;
-  static constexpr int N_BARS = 13;
+  static constexpr int OFF_Q = 0;                     // the pair's Q tiles (one stage)
+  static constexpr int OFF_K = kHeadSlots * TILE_BYTES;   // 2 stages of k_bar chunks
+  static constexpr int OFF_STASH = OFF_K + 2 * TILE_BYTES;   // [32][256] fp32: a group's u, per row thread
+  static constexpr int OFF_BAR = OFF_STASH + 32 * kRows * kHeadSlots * 4;
+  static constexpr int B_QF = 0, B_QE = 1, B_KF = 2, B_KE = 4, B_SF = 6, B_SE = 8, B_DRAIN = 10;
+  static constexpr int N_BARS = 11;
   static constexpr int OFF_MISC = OFF_BAR + N_BARS * 8;
   static constexpr int SMEM_BYTES = OFF_MISC + 16 + 1024;
-  static constexpr int TMEM_COLS = 256;
+  static constexpr int TMEM_COLS = 2 * kHeadSlots * kCols;   // 2 buffers x 2 heads
   static_assert(SMEM_BYTES <= 232448, "shared memory budget");
 };
 
@@ -138,10 +141,13 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
   };
   const int nh_max = n_hist(rt.local0 + rt.q_len - 1);
   const int n_ch = (nh_max + kCols - 1) / kCols;
-  const int n_steps = gq * kPasses * n_ch;       // step t: head t / (kPasses n_ch), pass (t / n_ch) % kPasses, chunk t % n_ch
+  const int n_pairs = (gq + kHeadSlots - 1) / kHeadSlots;
+  const int per_pair = kPasses * n_ch;
+  const int n_steps = n_pairs * per_pair;        // step t: pair t / per_pair, pass (t / n_ch) % kPasses, chunk t % n_ch
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < C::N_BARS; ++i) ptx::mbar_init(bar(i), (i == C::B_SE || i == C::B_SE + 1) ? kRows : 1u);
+    for (int i = 0; i < C::N_BARS; ++i)
+      ptx::mbar_init(bar(i), (i == C::B_SE || i == C::B_SE + 1) ? kRows * kHeadSlots : 1u);
     *abort_flag = 0;
     ptx::fence_mbar_init();
   }
@@ -158,21 +164,23 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
     const uint64_t pol = ptx::l2_policy_evict_last();
     uint32_t leader = 0;
     bool ok = true;
-    int nq = 0, nk = 0;
+    int nq = 0, nk = 0;                          // Q (per pair) and k_bar loads issued
     for (int t = 0; ok && t < n_steps; ++t) {
-      const int hh = t / (kPasses * n_ch), ch = t % n_ch;
-      if (t % (kPasses * n_ch) == 0) {           // the head's Q tile, once per head
-        const int qs = nq % 2;
-        if (nq >= 2 && !warp_wait(bar(C::B_QE + qs), ((nq - 2) / 2) & 1, abort_flag)) {
+      const int pair = t / per_pair, ch = t % n_ch;
+      if (t % per_pair == 0) {                   // the pair's Q tiles, once per pair
+        if (pair >= 1 && !warp_wait(bar(C::B_QE), (pair - 1) & 1, abort_flag)) {
           ok = false;
           break;
         }
+        const int nheads = min(kHeadSlots, gq - pair * kHeadSlots);
         if (ptx::elect_one(leader)) {
-          ptx::mbar_arrive_expect_tx(bar(C::B_QF + qs), C::TILE_BYTES);
+          ptx::mbar_arrive_expect_tx(bar(C::B_QF), nheads * C::TILE_BYTES);
+          for (int sl = 0; sl < nheads; ++sl) {
 #pragma unroll
-          for (int kb = 0; kb < C::KB; ++kb)
-            ptx::tma_load_3d(sbase + C::OFF_Q + qs * C::TILE_BYTES + kb * C::BLOCK, &L.tm_q, bar(C::B_QF + qs),
-                             kb * 64, g * gq + hh, rt.q_start, pol);
+            for (int kb = 0; kb < C::KB; ++kb)
+              ptx::tma_load_3d(sbase + C::OFF_Q + sl * C::TILE_BYTES + kb * C::BLOCK, &L.tm_q, bar(C::B_QF),
+                               kb * 64, g * gq + pair * kHeadSlots + sl, rt.q_start, pol);
+          }
         }
         __syncwarp();
         ++nq;
@@ -193,9 +201,9 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
       ++nk;
     }
     if (!ok && lane == 0) record_failure(abort_flag, L.status);
+    // no copy in flight at exit: the last Q and k_bar loads have landed
     const volatile int never = 0;
-    for (int s = 0; s < 2 && s < nq; ++s)
-      ptx::mbar_wait(bar(C::B_QF + s), ((nq - 1 - s) / 2) & 1, &never, kWaitTimeoutNs);
+    if (nq > 0) ptx::mbar_wait(bar(C::B_QF), (nq - 1) & 1, &never, kWaitTimeoutNs);
     for (int s = 0; s < 2 && s < nk; ++s)
       ptx::mbar_wait(bar(C::B_KF + s), ((nk - 1 - s) / 2) & 1, &never, kWaitTimeoutNs);
   } else if (warp == kWarpMma) {
@@ -203,14 +211,11 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
     uint32_t leader = 0;
     int first_leader = -1;
     bool same = true, issued = false, ok = true;
-    int nq = 0;
     for (int t = 0; ok && t < n_steps; ++t) {
-      const int b = t % 2;
-      const bool head_start = t % (kPasses * n_ch) == 0;
-      const bool head_end = t % (kPasses * n_ch) == kPasses * n_ch - 1;
-      if (head_start) ++nq;
-      const int qs = (nq - 1) % 2;
-      if ((head_start && !warp_wait(bar(C::B_QF + qs), ((nq - 1) / 2) & 1, abort_flag)) ||
+      const int b = t % 2, pair = t / per_pair;
+      const bool pair_start = t % per_pair == 0;
+      const bool pair_end = t % per_pair == per_pair - 1;
+      if ((pair_start && !warp_wait(bar(C::B_QF), pair & 1, abort_flag)) ||
           !warp_wait(bar(C::B_KF + t % 2), (t / 2) & 1, abort_flag) ||
           (t >= 2 && !warp_wait(bar(C::B_SE + b), ((t - 2) / 2) & 1, abort_flag))) {
         ok = false;
@@ -221,17 +226,20 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
       if (first_leader < 0) first_leader = static_cast<int>(leader);
       same = same && static_cast<int>(leader) == first_leader;
       if (me && same) {
-        const uint32_t qbase = sbase + C::OFF_Q + qs * C::TILE_BYTES;
+        const int nheads = min(kHeadSlots, gq - pair * kHeadSlots);
         const uint32_t kbase = sbase + C::OFF_K + (t % 2) * C::TILE_BYTES;
+        for (int sl = 0; sl < nheads; ++sl) {
+          const uint32_t qbase = sbase + C::OFF_Q + sl * C::TILE_BYTES;
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t a = ptx::sdesc_sw128(qbase + (kk / 4) * C::BLOCK + (kk % 4) * 32, 16, 1024);
-          const uint64_t bd = ptx::sdesc_sw128(kbase + (kk / 4) * C::BLOCK + (kk % 4) * 32, 16, 1024);
-          ptx::mma_ss(tmem + b * kCols, a, bd, kIdesc, kk > 0 ? 1u : 0u);
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint64_t a = ptx::sdesc_sw128(qbase + (kk / 4) * C::BLOCK + (kk % 4) * 32, 16, 1024);
+            const uint64_t bd = ptx::sdesc_sw128(kbase + (kk / 4) * C::BLOCK + (kk % 4) * 32, 16, 1024);
+            ptx::mma_ss(tmem + (b * kHeadSlots + sl) * kCols, a, bd, kIdesc, kk > 0 ? 1u : 0u);
+          }
         }
         ptx::mma_commit(bar(C::B_SF + b));
         ptx::mma_commit(bar(C::B_KE + t % 2));
-        if (head_end) ptx::mma_commit(bar(C::B_QE + qs));
+        if (pair_end) ptx::mma_commit(bar(C::B_QE));
       }
       __syncwarp();
       issued = true;
@@ -249,16 +257,19 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
     __syncwarp();
   } else {
     // Row threads: row = TMEM lane; the row's video-local position and |H_i|.
-    const int row = threadIdx.x;
+    const int slot = warp / 4, row = threadIdx.x % kRows;
     const bool row_ok = row < rt.q_len;
     const int pos = rt.local0 + row;
     const int nh = row_ok ? n_hist(pos) : 0;
-    const uint32_t tbase = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    const uint32_t tbase = tmem + (static_cast<uint32_t>((warp % 4) * 32) << 16) + slot * kCols;
     const float sc = L.scale_log2;               // logits in log2 units
-    float* stash = reinterpret_cast<float*>(smem + C::OFF_STASH) + row;   // this row's column: stash[e * 128]
+    constexpr int kStash = kRows * kHeadSlots;   // this thread's column: stash[e * kStash]
+    float* stash = reinterpret_cast<float*>(smem + C::OFF_STASH) + slot * kRows + row;
     bool ok = true;
-    for (int hh = 0; hh < gq; ++hh) {
-      const int h = g * gq + hh;
+    for (int pair = 0; pair < n_pairs; ++pair) {
+      const int hh = pair * kHeadSlots + slot;
+      const bool active = hh < gq;               // warp-uniform: an odd group leaves the last slot idle
+      const int h = g * gq + min(hh, gq - 1);
       float m = -INFINITY, gmin = INFINITY, z = 0.f;
       float inv_r = 0.f, target = 0.f, above = 0.f, tie = 0.f;
       int wkey = 0;                              // the boundary's key digits found so far
@@ -276,9 +287,9 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
 #pragma unroll
         for (int k = 0; k < kDigBins; ++k) acc[k] = 0.f;
         for (int ch = 0; ch < n_ch; ++ch) {
-          const int t = (hh * kPasses + pass) * n_ch + ch, b = t % 2;
+          const int t = (pair * kPasses + pass) * n_ch + ch, b = t % 2;
           ok = ok && warp_wait(bar(C::B_SF + b), (t / 2) & 1, abort_flag);
-          if (ok && __any_sync(0xffffffffu, nh > ch * kCols)) {   // warp-uniform: tcgen05.ld is collective
+          if (ok && active && __any_sync(0xffffffffu, nh > ch * kCols)) {   // warp-uniform: tcgen05.ld is collective
             ptx::tc_fence_after();
             // One compact loop per pass (uniform over the warp), 32 columns at a
             // time. x, the key and the weight use non-contracted arithmetic so
@@ -286,7 +297,7 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
 #pragma unroll 1
             for (int c0 = 0; c0 < kCols; c0 += 32) {
               uint32_t r[32];
-              ptx::tmem_ld32(tbase + b * kCols + c0, r);
+              ptx::tmem_ld32(tbase + b * kHeadSlots * kCols + c0, r);
               ptx::tmem_wait_ld();
               const int jn = nh - (ch * kCols + c0);         // columns e < jn are in H_i
               if (pass == 0) {
@@ -333,13 +344,13 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
                   const float v = __fmul_rn(u, inv_r);
                   if (e < jn && v >= lo && v < hi) {
                     in_mask |= 1u << e;
-                    stash[e * kRows] = u;
+                    stash[e * kStash] = u;
                   }
                 }
                 while (in_mask != 0u) {
                   const int e = __ffs(in_mask) - 1;
                   in_mask &= in_mask - 1u;
-                  const float u = stash[e * kRows];
+                  const float u = stash[e * kStash];
                   const int key = min(kQMax, __float2int_rz(__fmul_rn(u, inv_r)));
                   bin_add<0, 16>(acc, (key >> dshift) & ((1 << width) - 1), ptx::ex2(-u));
                 }
@@ -356,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
                   word |= (e < jn && v < k0) ? 1u << e : 0u;
                   if (e < jn && v >= k0 && v < k1) {
                     at_mask |= 1u << e;
-                    stash[e * kRows] = u;
+                    stash[e * kStash] = u;
                   }
                 }
                 // the boundary key: lower ids first while the mass before them is below the target
@@ -364,7 +375,7 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
                   const int e = __ffs(at_mask) - 1;
                   at_mask &= at_mask - 1u;
                   if (above + tie < target) word |= 1u << e;
-                  tie += ptx::ex2(-stash[e * kRows]);
+                  tie += ptx::ex2(-stash[e * kStash]);
                 }
                 __syncwarp();
                 const int w = ch * 4 + (c0 >> 5);
@@ -375,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
               }
             }
             ptx::tc_fence_before();
-          } else if (pass == kPasses - 1 && row_ok && ok) {
+          } else if (pass == kPasses - 1 && row_ok && ok && active) {
             // No column of this chunk is in H_i for the warp: zeros (and the own block).
             for (int wi = 0; wi < 4; ++wi) {
               const int w = ch * 4 + wi;
@@ -413,7 +424,7 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
         }
       }
       // The own block's word when it lies past the chunks of this tile.
-      if (row_ok && ok && (nh >> 5) >= n_ch * 4 && (nh >> 5) < L.n_words)
+      if (row_ok && ok && active && (nh >> 5) >= n_ch * 4 && (nh >> 5) < L.n_words)
         keep[static_cast<int64_t>(nh >> 5) * L.n_tok] = 1u << (nh & 31);
     }
     if (!ok && row == 0) record_failure(abort_flag, L.status);
