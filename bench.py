@@ -509,6 +509,7 @@ def bench_ours(args, cfg):
                 "tokens_per_s": world * st["n_tok"] * cfg.layers / (ms_step * 1e-3),
                 "flop_per_step": st["flop"], "flop_causal_valid_per_step": st["flop_valid"],
                 "attention": {"ms": attn_avg, "tflops": attn_tflops, "frac_of_bf16_peak": attn_tflops / peaks["bf16"],
+                              "frac_of_bf16_sustained": attn_tflops / peaks["bf16_sus"],
                               "tflops_causal_valid": st["flop_valid"] / (attn_avg * 1e-3) / 1e12},
                 "evidence": {"ms": ev_avg, "gbs": ev_gbs, "frac_of_hbm": ev_gbs / peaks["hbm"],
                              "bytes": st["evidence_bytes"]},
