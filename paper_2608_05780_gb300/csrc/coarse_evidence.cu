@@ -7,11 +7,15 @@
 // visual tokens m, frame sums, head sums and A_qf. All tokens of a retained
 // visual block share its weight exp(g_ij - M_i) / Z_i.
 //
-// coarse_rows_kernel: one warp per (text row, head). Lanes split d; for every
-//   block of the row's history the warp forms g_ij (stored for the next
-//   kernel) and, over S_i (the keep bits), the running max M_i and the sum
-//   Z_i = sum_{S_i} B exp(g - M) + sum_{E_i} exp(s - M) with the exact own-block
-//   logits s.
+// coarse_rows_kernel: one CTA per (8 text rows of a video, head), a warp per
+//   row. The CTA stages the k_bar rows of the head's KV group in chunks of 32
+//   blocks (one keep word) in shared memory; lane j of a warp takes block
+//   j of each chunk: it forms g_ij = scale q_i k_bar_j (stored for the next
+//   kernel) and, over its blocks in S_i, a running max and sum. The lanes'
+//   pairs then merge (a butterfly: each step's merge is symmetric, so all
+//   lanes agree) and the warp adds the exact logits s of the own block's
+//   causal prefix E_i, giving M_i and
+//   Z_i = sum_{S_i} B exp(g - M) + sum_{E_i} exp(s - M).
 // coarse_map_kernel: one thread per (frame, head, video): for each block of
 //   the frame, c_j = sum over the video's text rows of [j in S_i]
 //   exp(g_ij - M_i) / Z_i (rows in order: deterministic); writes c_j to the
@@ -35,53 +39,107 @@ __device__ __forceinline__ float warp_sum(float x) {
   return x;
 }
 
+// s + sum of the 8 bf16 products of a and b, in order.
+__device__ __forceinline__ float dot8(const uint4& a, const uint4& b, float s) {
+  const __nv_bfloat162* a2 = reinterpret_cast<const __nv_bfloat162*>(&a);
+  const __nv_bfloat162* b2 = reinterpret_cast<const __nv_bfloat162*>(&b);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 fa = __bfloat1622float2(a2[i]), fb = __bfloat1622float2(b2[i]);
+    s = fmaf(fa.x, fb.x, s);
+    s = fmaf(fa.y, fb.y, s);
+  }
+  return s;
+}
+
+// (m, z) <- the softmax pair of (m, z) and (m2, z2): max and rescaled sum.
+__device__ __forceinline__ void merge_mz(float& m, float& z, float m2, float z2) {
+  const float mm = fmaxf(m, m2);
+  z = mm == -INFINITY ? 0.f : z * __expf(m - mm) + z2 * __expf(m2 - mm);
+  m = mm;
+}
+
+constexpr int kRowsPerCta = 8;                   // text rows (warps) per CTA
+constexpr int kChunk = 32;                       // k_bar rows staged at a time: one keep word
+
 __global__ void __launch_bounds__(256) coarse_rows_kernel(const __grid_constant__ CoarseLaunch L) {
-  const int warp_global = blockIdx.x * 8 + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
+  __shared__ __align__(16) __nv_bfloat16 q_s[kRowsPerCta][128];   // each warp's query row
+  __shared__ uint4 kb_s[kChunk][128 / 8 + 1];                     // k_bar rows, padded by 16 B
+  const int wib = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
-  if (warp_global >= L.total_text) return;       // warp-uniform
-  // The text row: find its video (text rows of the videos back to back).
-  int v = 0;
-  while (v + 1 < L.n_videos && L.text_off[v + 1] <= warp_global) ++v;
+  // This CTA's video and row group (groups of 8 text rows, videos back to back).
+  int v = 0, grp = blockIdx.x;
+  for (; v < L.n_videos; ++v) {
+    const int cnt = (L.text_off[v + 1] - L.text_off[v] + kRowsPerCta - 1) / kRowsPerCta;
+    if (grp < cnt) break;
+    grp -= cnt;
+  }
+  if (v >= L.n_videos) return;                   // CTA-uniform, before any barrier
   const ToppVideo vid = L.vids[v];
-  const int t = warp_global - L.text_off[v];     // text row within the video
+  const int n_text = L.text_off[v + 1] - L.text_off[v];
+  const int t_last = min(grp * kRowsPerCta + kRowsPerCta - 1, n_text - 1);
+  const int t = min(grp * kRowsPerCta + wib, t_last);   // text row within the video (clamped)
+  const bool active = grp * kRowsPerCta + wib <= t_last;   // warp-uniform
+  const int trow = L.text_off[v] + t;            // text row over all videos
   const int pos = vid.n_vis + t;                 // video-local position
   const int row = vid.start + pos;               // global token
   const int B = L.block, nvb = vid.n_vis / B;
   const int nh = nvb + t / B;                    // blocks that end before the row
+  const int nh_cta = nvb + t_last / B;           // the most over the CTA's rows
   const int own0 = vid.n_vis + (t / B) * B;      // first token of its own block
   const int g = h / (L.hq / L.hkv);
-  const int d = L.head_dim;
+  const int d = L.head_dim, dc = d / 8;          // d = 64 or 128
   const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(L.q) + (static_cast<int64_t>(row) * L.hq + h) * d;
+  for (int c = lane; c < dc; c += 32) reinterpret_cast<uint4*>(q_s[wib])[c] = reinterpret_cast<const uint4*>(q)[c];
+  __syncwarp();
+  const uint4* q4 = reinterpret_cast<const uint4*>(q_s[wib]);
   const __nv_bfloat16* kbar = static_cast<const __nv_bfloat16*>(L.kbar);
   const __nv_bfloat16* k = static_cast<const __nv_bfloat16*>(L.k);
-  // This lane's d / 32 query elements (d = 64 or 128: 2 or 4 per lane).
-  float qv[4] = {0.f, 0.f, 0.f, 0.f};
-  const int per = d / 32;
-  for (int e = 0; e < per; ++e) qv[e] = __bfloat162float(q[lane * per + e]);
-  auto dot = [&](const __nv_bfloat16* kr) {
-    float s = 0.f;
-    for (int e = 0; e < per; ++e) s += qv[e] * __bfloat162float(kr[lane * per + e]);
-    return warp_sum(s) * L.scale;
-  };
-  float* grow = L.gbuf + (static_cast<int64_t>(h) * L.total_text + warp_global) * L.pitch;
+  float* grow = L.gbuf + (static_cast<int64_t>(h) * L.total_text + trow) * L.pitch;
   const uint32_t* keep = L.keep + static_cast<int64_t>(h) * L.n_words * L.n_tok + row;
   float m = -INFINITY, z = 0.f;
-  uint32_t word = 0u;
-  for (int j = 0; j < nh; ++j) {
-    if ((j & 31) == 0) word = keep[static_cast<int64_t>(j >> 5) * L.n_tok];
-    const float gj = dot(kbar + (static_cast<int64_t>(vid.blk_off + j) * L.hkv + g) * d);
-    if (lane == 0) grow[j] = gj;
-    if ((word >> (j & 31)) & 1u) {               // j in S_i: B tokens share g_ij
-      if (gj > m) {
-        z = (m == -INFINITY) ? 0.f : z * __expf(m - gj);
-        m = gj;
+  for (int j0 = 0; j0 < nh_cta; j0 += kChunk) {
+    __syncthreads();                             // the previous chunk is consumed
+    for (int i = threadIdx.x; i < kChunk * dc; i += blockDim.x) {   // coalesced: 16 B per thread
+      const int jj = i / dc, c = i % dc;
+      if (j0 + jj < nh_cta)
+        kb_s[jj][c] = reinterpret_cast<const uint4*>(kbar + (static_cast<int64_t>(vid.blk_off + j0 + jj) * L.hkv + g) * d)[c];
+    }
+    __syncthreads();
+    const int j = j0 + lane;
+    if (active && j < nh) {
+      const uint32_t word = keep[static_cast<int64_t>(j0 >> 5) * L.n_tok];
+      float s = 0.f;
+      for (int c = 0; c < dc; ++c) s = dot8(q4[c], kb_s[lane][c], s);
+      const float gj = s * L.scale;
+      grow[j] = gj;
+      if ((word >> lane) & 1u) {                 // j in S_i: B tokens share g_ij
+        if (gj > m) {
+          z = (m == -INFINITY) ? 0.f : z * __expf(m - gj);
+          m = gj;
+        }
+        z += static_cast<float>(B) * __expf(gj - m);
       }
-      z += static_cast<float>(B) * __expf(gj - m);
     }
   }
-  for (int mm = own0; mm <= pos; ++mm) {          // E_i: exact logits of the own block's causal prefix
-    const float s = dot(k + (static_cast<int64_t>(vid.start + mm) * L.hkv + g) * d);
+  if (!active) return;                           // warp-uniform; no barrier follows
+  for (int off = 16; off > 0; off >>= 1) {
+    const float m2 = __shfl_xor_sync(kFull, m, off), z2 = __shfl_xor_sync(kFull, z, off);
+    merge_mz(m, z, m2, z2);
+  }
+  // E_i: exact logits of the own block's causal prefix; lanes split d.
+  const int per = d / 32;
+  float qv[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int e = 0; e < 4; ++e)
+    if (e < per) qv[e] = __bfloat162float(q_s[wib][lane * per + e]);
+  for (int mm = own0; mm <= pos; ++mm) {
+    const __nv_bfloat16* kr = k + (static_cast<int64_t>(vid.start + mm) * L.hkv + g) * d;
+    float s = 0.f;
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      if (e < per) s += qv[e] * __bfloat162float(kr[lane * per + e]);
+    s = warp_sum(s) * L.scale;
     if (s > m) {
       z = (m == -INFINITY) ? 0.f : z * __expf(m - s);
       m = s;
@@ -89,8 +147,8 @@ __global__ void __launch_bounds__(256) coarse_rows_kernel(const __grid_constant_
     z += __expf(s - m);
   }
   if (lane == 0) {
-    L.row_m[static_cast<int64_t>(h) * L.total_text + warp_global] = m;
-    L.row_z[static_cast<int64_t>(h) * L.total_text + warp_global] = z;
+    L.row_m[static_cast<int64_t>(h) * L.total_text + trow] = m;
+    L.row_z[static_cast<int64_t>(h) * L.total_text + trow] = z;
   }
 }
 
@@ -148,7 +206,7 @@ __global__ void __launch_bounds__(128) coarse_finalize_kernel(const __grid_const
 cudaError_t launch_coarse(const CoarseLaunch& L, cudaStream_t stream) {
   if (L.n_videos == 0) return cudaSuccess;
   if (L.total_text > 0) {
-    dim3 g1((L.total_text + 7) / 8, L.hq);
+    dim3 g1(L.row_groups, L.hq);
     coarse_rows_kernel<<<g1, 256, 0, stream>>>(L);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
