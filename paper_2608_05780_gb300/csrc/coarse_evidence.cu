@@ -206,7 +206,9 @@ __global__ void __launch_bounds__(128) coarse_finalize_kernel(const __grid_const
 cudaError_t launch_coarse(const CoarseLaunch& L, cudaStream_t stream) {
   if (L.n_videos == 0) return cudaSuccess;
   if (L.total_text > 0) {
-    dim3 g1(L.row_groups, L.hq);
+    // groups of 8 text rows per video: at most total_text / 8 + one partial group per video;
+    // CTAs past the last group return at once
+    dim3 g1((L.total_text + 7) / 8 + L.n_videos, L.hq);
     coarse_rows_kernel<<<g1, 256, 0, stream>>>(L);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;

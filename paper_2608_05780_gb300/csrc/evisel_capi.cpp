@@ -929,11 +929,10 @@ int evisel_coarse_evidence(const evisel_probe_args* a, evisel_ws* ws, int32_t bl
   if (a->num_videos == 0) return EVISEL_OK;
   const int npf = a->tokens_per_frame;
   std::vector<int> text_off(1, 0), vis_off(1, 0), frame_off(1, 0);
-  int max_frames = 0, row_groups = 0;
+  int max_frames = 0;
   for (int b = 0; b < a->num_videos; ++b) {
     const int nv = a->n_vis_h[b], nt = a->cu_seqlens_h[b + 1] - a->cu_seqlens_h[b] - nv;
     text_off.push_back(text_off.back() + nt);
-    row_groups += (nt + 7) / 8;                  // CTAs of the coarse rows kernel
     vis_off.push_back(vis_off.back() + nv);
     frame_off.push_back(frame_off.back() + nv / npf);
     max_frames = std::max(max_frames, nv / npf);
@@ -996,7 +995,6 @@ int evisel_coarse_evidence(const evisel_probe_args* a, evisel_ws* ws, int32_t bl
   L.total_vis = vis_off.back();
   L.total_frames = frame_off.back();
   L.max_frames = max_frames;
-  L.row_groups = row_groups;
   L.accumulate = accumulate != 0;
   L.scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / std::sqrt(float(a->head_dim));
   e = launch_coarse(L, stream);

@@ -242,7 +242,6 @@ struct CoarseLaunch {
   float* aqf;
   int n_videos, total_text, pitch, n_words, n_tok, hq, hkv, head_dim, block, tokens_per_frame;
   int total_vis, total_frames, max_frames, accumulate;
-  int row_groups;                   // sum over videos of ceil(n_text / 8)
   float scale;
 };
 
