@@ -221,6 +221,26 @@ def bench_reference(args, cfg):
     return 0
 
 
+def _max_over_ranks(x, world):
+    """x at one rank; else the largest x over the ranks (the slowest rank's
+    time), by an all-reduce on the process group's device (CUDA under NCCL,
+    the host under gloo)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _whole_job_tflops(world, flop_per_replica_step, ms_per_step):
+    """Whole-job throughput: one step's FLOP on every replica over the
+    (max-over-ranks) step time."""
+    return world * flop_per_replica_step / (ms_per_step * 1e-3) / 1e12
+
+
 def _config_dict(cfg, st):
     return {"workload": f"{cfg.name}: {cfg.description}", "tokens": st["n_tok"], "kept_tiles": st["tiles"],
             "layers": cfg.layers, "videos": cfg.num_videos, "hq": cfg.hq, "hkv": cfg.hkv,
@@ -293,12 +313,9 @@ def bench_ours(args, cfg):
     elapsed_ms = t_start.elapsed_time(t_end)
     attn_ms = [m[0].elapsed_time(m[1]) for m in marks]
     ev_ms = [m[1].elapsed_time(m[2]) for m in marks]
-    if world > 1:
-        t = torch.tensor([elapsed_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = _max_over_ranks(elapsed_ms, world)
     ms_step = elapsed_ms / args.steps
-    value = world * st["flop"] / (ms_step * 1e-3) / 1e12
+    value = _whole_job_tflops(world, st["flop"], ms_step)
     attn_avg = sum(attn_ms) / len(attn_ms)
     ev_avg = sum(ev_ms) / len(ev_ms)
     peaks = _peaks()
@@ -356,13 +373,15 @@ def bench_ours(args, cfg):
 
     e2e_run(max(1, args.warmup))
     torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     e2e_run(args.steps, start_evt=e0)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1) / args.steps
+    e2e_ms = _max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     # the copies are done: the last step's maps are on the host
     if not all(np.isfinite(hm.numpy()).all() for hm in host_maps):
         raise RuntimeError("non-finite evidence maps")
@@ -532,7 +551,7 @@ def bench_ours(args, cfg):
                                 "probe_overhead_ms": pcf_ms - attn_avg,
                                 "ms": cf_ms, "gbs": cf_bytes / (cf_ms * 1e-3) / 1e9,
                                 "frac_of_hbm": cf_bytes / (cf_ms * 1e-3) / 1e9 / peaks["hbm"], "bytes": cf_bytes},
-                "e2e": {"value": world * st["flop"] / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+                "e2e": {"value": _whole_job_tflops(world, st["flop"], e2e_ms), "unit": "TFLOP/s",
                         "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
                 "gpu_launches": args.steps * (4 if _has_combine(probe) else 3),
                 "clocks": clk}
