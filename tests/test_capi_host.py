@@ -141,3 +141,38 @@ def test_binding_fails_loudly_without_library(tmp_path):
             B.load(str(tmp_path / "missing.so"))
     finally:
         B._lib = saved
+
+
+@pytest.mark.parametrize("block,tau,over,code", [
+    (24, 0.97, {}, -2),                  # block not a power of two
+    (8, 0.97, {}, -2),                   # block below 16
+    (32, 0.97, {}, -2),                  # block above N_v (16): it must divide the frames
+    (16, 0.0, {}, -1),                   # tau_p outside (0, 1]
+    (16, 1.5, {}, -1),
+    (16, float("nan"), {}, -1),
+    (16, 0.97, dict(q=FAKE + 8), -1),    # q not 16-byte aligned (TMA)
+    (16, 0.97, dict(d=96), -2),
+    (16, 0.97, dict(hq=5, hkv=2), -2),
+    (16, 0.97, dict(n_vis=[250]), -1),   # n_vis not a multiple of N_v
+    (16, 0.97, dict(scale=-1.0), -1),
+])
+def test_topp_validation_rejects(lib, block, tau, over, code):
+    a, keep = _args(**over)
+    ws = ctypes.c_void_p(None)
+    rc = lib.evisel_topp_mask(ctypes.byref(a), block, tau, ctypes.c_void_p(FAKE), None, None, ctypes.byref(ws))
+    assert rc == code, lib.evisel_last_error()
+    assert ws.value is None          # nothing allocated, nothing launched
+    assert lib.evisel_last_error()
+
+
+def test_topp_null_keep_and_workspace_pointer(lib):
+    a, keep = _args()
+    ws = ctypes.c_void_p(None)
+    assert lib.evisel_topp_mask(ctypes.byref(a), 16, 0.97, None, None, None, ctypes.byref(ws)) == -1
+    assert lib.evisel_topp_mask(ctypes.byref(a), 16, 0.97, ctypes.c_void_p(FAKE), None, None, None) == -1
+
+
+def test_coarse_evidence_without_workspace(lib):
+    a, keep = _args()
+    fake = ctypes.c_void_p(FAKE)
+    assert lib.evisel_coarse_evidence(ctypes.byref(a), None, 16, fake, fake, fake, fake, fake, 0, None) == -1
