@@ -24,6 +24,7 @@
 #include <string>
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "../../include/evisel.h"
 #include "evisel_internal.h"
@@ -174,6 +175,10 @@ void make_plan(const evisel_probe_args* a, Counts& c, const Out* o) {
 
 extern "C" int evisel_probe_evidence_noalloc(const evisel_probe_args* args, float* tok, float* frame, float* head,
                                              float* aqf, int accumulate, void* stream_ptr, int* device_status) {
+  nvtxRangePushA("evisel_probe_evidence_noalloc");
+  struct Pop {
+    ~Pop() { nvtxRangePop(); }
+  } const nvtx_pop;
   clear_last_error();
   int rc = validate_probe_args(args);
   if (rc != EVISEL_OK) return rc;
