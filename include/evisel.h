@@ -38,7 +38,9 @@ extern "C" {
 #define EVISEL_ECUDA         -4  /* a CUDA runtime/driver call failed             */
 #define EVISEL_ENOMEM        -5  /* device or pinned allocation failed            */
 #define EVISEL_ETIMEOUT      -6  /* device-side: a bounded wait gave up           */
-#define EVISEL_EBOUNDS       -7  /* device-side: an index check failed            */
+#define EVISEL_EBOUNDS       -7  /* reserved for device-side index checks; every index is
+                                     validated on the host before launch, and no kernel of
+                                     this library records it */
 #define EVISEL_ESTATE        -8  /* evidence requested before any probe on the workspace */
 
 /* Opaque workspace owned by the library: work list, device copy of the mask,
@@ -148,7 +150,8 @@ int evisel_evidence_reduce(const evisel_ws* ws, float* tok, float* frame, float*
 void evisel_free(evisel_ws* ws);
 
 /* Synchronises the stream of the workspace's last call and returns the device
- * status word (EVISEL_OK, EVISEL_ETIMEOUT or EVISEL_EBOUNDS), then clears it.
+ * status word (EVISEL_OK or EVISEL_ETIMEOUT; EVISEL_EBOUNDS is reserved), then
+ * clears it.
  * Returns EVISEL_ECUDA if the synchronisation itself failed. */
 int evisel_status(evisel_ws* ws);
 
