@@ -164,6 +164,12 @@ const char* evisel_last_error(void);
 /* Bytes of device memory currently held by the workspace (0 for NULL). */
 int64_t evisel_workspace_bytes(const evisel_ws* ws);
 
+/* Identity of this binary: a hash of the sources, headers, compiler flags,
+ * compiler version and machine type it was built from (a static string owned
+ * by the library). The paper has no counterpart; it lets a log show which
+ * build ran. */
+const char* evisel_build_id(void);
+
 /* ---- Entry point that allocates nothing ---------------------------------------
  * The paper has no counterpart to this call. It serves callers of this library
  * that cannot call cudaMalloc on their serving path: servers that hand all device

@@ -12,8 +12,14 @@ from ._binding import (  # noqa: F401
 )
 
 
-def ensure_built():
-    """Builds the library if needed and loads it."""
+def ensure_built(verbose: bool = True):
+    """Builds the library if it does not hold the current tree's build id,
+    loads it, and (``verbose``) reports the id of the binary that loaded."""
+    import sys
+
     from .build import build
-    build()
-    return load()
+    path = build()
+    lib = load()
+    if verbose:
+        sys.stderr.write(f"libevisel.so build {lib.evisel_build_id().decode()} ({path})\n")
+    return lib

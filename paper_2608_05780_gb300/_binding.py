@@ -53,7 +53,7 @@ class ProbeArgs(ctypes.Structure):
 
 
 EXPORTS = ["evisel_probe_attention", "evisel_evidence_reduce", "evisel_free", "evisel_status",
-           "evisel_strerror", "evisel_last_error", "evisel_workspace_bytes"]
+           "evisel_strerror", "evisel_last_error", "evisel_workspace_bytes", "evisel_build_id"]
 
 _lib = None
 
@@ -81,6 +81,8 @@ def load(path: str = LIB_PATH):
     lib.evisel_last_error.restype = ctypes.c_char_p
     lib.evisel_workspace_bytes.argtypes = [vp]
     lib.evisel_workspace_bytes.restype = ctypes.c_int64
+    lib.evisel_build_id.argtypes = []
+    lib.evisel_build_id.restype = ctypes.c_char_p
     lib.evisel_probe_evidence_noalloc.argtypes = [ctypes.POINTER(ProbeArgs), vp, vp, vp, vp, i32, vp,
                                                   ctypes.POINTER(ctypes.c_int)]
     lib.evisel_probe_evidence_noalloc.restype = i32

@@ -1073,6 +1073,14 @@ const char* evisel_strerror(int code) {
 
 const char* evisel_last_error(void) { return g_last_error.c_str(); }
 
+#ifndef EVISEL_BUILD_ID
+#define EVISEL_BUILD_ID "unversioned"
+#endif
+// The prefix lets the build script find the id in the binary without loading it.
+static const char kBuildIdString[] = "evisel-build-id:" EVISEL_BUILD_ID;
+
+const char* evisel_build_id(void) { return kBuildIdString + sizeof("evisel-build-id:") - 1; }
+
 int64_t evisel_workspace_bytes(const evisel_ws* ws) {
   return ws ? static_cast<int64_t>(ws->arena_bytes) : 0;
 }

@@ -2,9 +2,11 @@
 // sm_103a kernels. Not part of the public ABI.
 #pragma once
 
+#include <atomic>
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <mutex>
 
 namespace evisel {
 
@@ -255,6 +257,27 @@ cudaError_t launch_evidence(const EvidenceLaunch& L, cudaStream_t stream);
 int encode_tensor_map(CUtensorMap* map, const void* base, int n_tok, int heads, int d, int rows);
 int set_last_error(int code, const char* msg);
 void clear_last_error();
+
+// A kernel's dynamic shared-memory limit is an attribute of the current
+// device: raise it once per device (ordinals below 64; others every launch),
+// under a lock so that concurrent first launches on one device agree.
+struct PerDeviceAttr {
+  std::atomic<uint64_t> done{0};
+  std::mutex mu;
+};
+
+inline cudaError_t raise_smem_limit(PerDeviceAttr& once, const void* kern, int bytes) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = dev < 64 ? (1ull << dev) : 0ull;
+  if (bit && (once.done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  std::lock_guard<std::mutex> lock(once.mu);
+  if (bit && (once.done.load(std::memory_order_relaxed) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && bit) once.done.fetch_or(bit, std::memory_order_release);
+  return e;
+}
 
 // Bounded waits give up after this many nanoseconds of %globaltimer.
 constexpr uint64_t kWaitTimeoutNs = 2000000000ull;

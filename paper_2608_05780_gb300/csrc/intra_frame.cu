@@ -388,12 +388,9 @@ template <int D, int W>
 cudaError_t launch_dw(const IntraFrameLaunch& L, cudaStream_t stream) {
   using C = IfCfg<D>;
   auto kern = intra_frame_kernel<D, W>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static PerDeviceAttr smem_once;
+  cudaError_t e = raise_smem_limit(smem_once, reinterpret_cast<const void*>(kern), C::SMEM_BYTES);
+  if (e != cudaSuccess) return e;
   const int n_sm = sm_count();
   if (n_sm <= 0) return cudaErrorInvalidDevice;
   const int grid = L.total_blocks < n_sm ? L.total_blocks : n_sm;

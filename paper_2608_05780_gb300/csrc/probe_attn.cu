@@ -580,46 +580,45 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
     ptx::mbar_arrive(bar_pf);
   }
 
-  if (!ok) {
-    record_failure(abort_flag, L.status, kStatusTimeout);
-    return;
-  }
-  if (!warp_wait(bar(C::B_OF + slot), 0, abort_flag)) {
-    record_failure(abort_flag, L.status, kStatusTimeout);
-    return;
-  }
+  ok = ok && warp_wait(bar(C::B_OF + slot), 0, abort_flag);
+  if (!ok) record_failure(abort_flag, L.status, kStatusTimeout);
   ptx::tc_fence_after();
 
   const float inv_l = l_sum > 0.f ? 1.f / l_sum : 0.f;
   if (it.part < 0 && it.q_len == TILE) {
+    // Every warp of the slot reaches the named barrier below, whether or not
+    // one of them gave up on a wait, so that the barrier always completes;
+    // the barrier then tells all 128 threads whether to store.
     // Full tile: the slot's O goes through its Q region of shared memory (no
     // MMA reads Q any more) in Q's swizzled layout, then out by TMA stores of
     // one 64-column block of one head each: whole 128-byte rows instead of 16
     // bytes per row and store.
     const uint32_t stage = sbase + C::OFF_Q + slot * C::Q_BYTES + hp * TILE * 128 + row_local * 128;
+    if (ok) {
 #pragma unroll
-    for (int c = 0; c < D / 32; ++c) {
-      uint32_t r[32];
-      ptx::tmem_ld32(tmem + C::COL_O + c * 32, r);
-      ptx::tmem_wait_ld();
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t r[32];
+        ptx::tmem_ld32(tmem + C::COL_O + c * 32, r);
+        ptx::tmem_wait_ld();
 #pragma unroll
-      for (int q4 = 0; q4 < 4; ++q4) {
-        uint4 w;
-        w.x = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 0]) * inv_l, __uint_as_float(r[8 * q4 + 1]) * inv_l);
-        w.y = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 2]) * inv_l, __uint_as_float(r[8 * q4 + 3]) * inv_l);
-        w.z = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 4]) * inv_l, __uint_as_float(r[8 * q4 + 5]) * inv_l);
-        w.w = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 6]) * inv_l, __uint_as_float(r[8 * q4 + 7]) * inv_l);
-        // 16-byte chunk k of the row's 128-byte block kb sits at chunk k ^ (row & 7).
-        const int kb = c / 2, k = (c % 2) * 4 + q4;
-        const uint32_t addr = stage + kb * C::Q_BLOCK + ((k ^ (row_local & 7)) << 4);
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
-                     : "memory");
+        for (int q4 = 0; q4 < 4; ++q4) {
+          uint4 w;
+          w.x = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 0]) * inv_l, __uint_as_float(r[8 * q4 + 1]) * inv_l);
+          w.y = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 2]) * inv_l, __uint_as_float(r[8 * q4 + 3]) * inv_l);
+          w.z = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 4]) * inv_l, __uint_as_float(r[8 * q4 + 5]) * inv_l);
+          w.w = ptx::pack_bf16x2(__uint_as_float(r[8 * q4 + 6]) * inv_l, __uint_as_float(r[8 * q4 + 7]) * inv_l);
+          // 16-byte chunk k of the row's 128-byte block kb sits at chunk k ^ (row & 7).
+          const int kb = c / 2, k = (c % 2) * 4 + q4;
+          const uint32_t addr = stage + kb * C::Q_BLOCK + ((k ^ (row_local & 7)) << 4);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
+                       : "memory");
+        }
       }
     }
-    if (row_ok) L.lse[static_cast<int64_t>(head) * L.n_tok + qpos] = (m_used + __log2f(l_sum)) * kLn2;
+    if (ok && row_ok) L.lse[static_cast<int64_t>(head) * L.n_tok + qpos] = (m_used + __log2f(l_sum)) * kLn2;
     ptx::fence_proxy_async_smem();
-    ptx::bar_sync(1 + slot, kRows);
-    if ((threadIdx.x & 127) == 0) {
+    const bool all_ok = ptx::bar_and(1 + slot, kRows, ok);
+    if (all_ok && (threadIdx.x & 127) == 0) {
 #pragma unroll
       for (int h = 0; h < C::HP; ++h) {
         if (slot * C::HP + h >= left) break;   // heads past the group's end are not stored
@@ -631,6 +630,8 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
       ptx::bulk_commit();
       ptx::bulk_wait_read();   // the shared memory source must outlive the copy
     }
+  } else if (!ok) {
+    return;
   } else if (it.part < 0) {
     uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(L.o) +
                                           (static_cast<int64_t>(qpos) * L.hq + head) * D);
@@ -719,12 +720,9 @@ cudaError_t launch_cfg(const ProbeLaunch& L, cudaStream_t stream) {
   constexpr int NS = 2;
   using C = Cfg<TILE, D, NS>;
   auto kern = probe_attn_kernel<TILE, D, NS, FSW, EMB>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static PerDeviceAttr smem_once;
+  cudaError_t e = raise_smem_limit(smem_once, reinterpret_cast<const void*>(kern), C::SMEM_BYTES);
+  if (e != cudaSuccess) return e;
   kern<<<L.n_items, kThreads, C::SMEM_BYTES, stream>>>(L);
   return cudaGetLastError();
 }

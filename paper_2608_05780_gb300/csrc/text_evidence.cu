@@ -255,12 +255,9 @@ template <int D>
 cudaError_t launch_d(const TextEvidenceLaunch& L, cudaStream_t stream) {
   using C = TeCfg<D>;
   auto kern = text_evidence_kernel<D>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static PerDeviceAttr smem_once;
+  cudaError_t e = raise_smem_limit(smem_once, reinterpret_cast<const void*>(kern), C::SMEM_BYTES);
+  if (e != cudaSuccess) return e;
   dim3 grid(L.n_chunks, L.hkv);
   kern<<<grid, kThreads, C::SMEM_BYTES, stream>>>(L);
   return cudaGetLastError();

@@ -483,12 +483,9 @@ template <int D>
 cudaError_t launch_select(const ToppLaunch& L, cudaStream_t stream) {
   using C = TpCfg<D>;
   auto kern = topp_select_kernel<D>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static PerDeviceAttr smem_once;
+  cudaError_t e = raise_smem_limit(smem_once, reinterpret_cast<const void*>(kern), C::SMEM_BYTES);
+  if (e != cudaSuccess) return e;
   dim3 grid(L.n_tiles, L.hkv);
   kern<<<grid, kThreads, C::SMEM_BYTES, stream>>>(L);
   return cudaGetLastError();

@@ -2,11 +2,17 @@
 binding and compare it with the float64 oracle at the stated tolerances.
 
 Tolerances (float64 oracle vs the bf16-in / bf16-out kernel):
-  O    max abs <= 2e-2 and relative L2 <= 5e-3
-  LSE  max abs <= 1e-3
-  maps token and frame maps divided by n_text (every entry <= 1): max abs <= 1e-3;
-       head map / n_text and A_qf: max abs <= 1e-3; identical planted top-k on the
-       head-summed frame map.
+  O      max abs <= 2e-2 and relative L2 <= 5e-3
+  LSE    max abs <= 1e-3
+  maps   frame map: max abs <= 1e-3 per entry, on the raw sums (over text
+         rows, and over layers where the maps accumulate), as the contract
+         states it for frame evidence; the token map at the same bound;
+         A_qf (an average over text rows and heads, summed over layers):
+         max abs <= 1e-3;
+         head map: relative error <= 1e-3 (each entry is a sum of
+         probabilities exp(s - LSE), so an LSE within 1e-3 moves it by at
+         most a factor e^(1e-3)); identical planted top-k on the head-summed
+         frame map.
 """
 import numpy as np
 
@@ -16,6 +22,7 @@ O_MAX_ABS = 2e-2
 O_REL_L2 = 5e-3
 LSE_ABS = 1e-3
 MAP_ABS = 1e-3
+HEAD_REL = 1e-3
 
 
 def to_device(probe):
@@ -71,24 +78,22 @@ def oracle_maps(probe):
     return oracle.evidence(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, probe.cfg.tokens_per_frame)
 
 
-def check_maps(gpu, ref, probe, layers=1, label=""):
-    """Compares maps normalised per text row (and per layer)."""
+def check_maps(gpu, ref, probe, label=""):
+    """Compares the raw maps (sums over layers on both sides where they accumulate)."""
     tok, frame, head, aqf = (np.asarray(x, np.float64) for x in gpu)
-    rtok, rframe, rhead, raqf = ref
+    rtok, rframe, rhead, raqf = (np.asarray(x, np.float64) for x in ref)
     cfg = probe.cfg
-    n_text = probe.n_text.astype(np.float64)
-    nvis = probe.n_vis
-    frames = nvis // cfg.tokens_per_frame
-    vis_cols = np.repeat(np.maximum(n_text, 1), nvis)
-    fr_cols = np.repeat(np.maximum(n_text, 1), frames)
-    e_tok = np.abs(tok - rtok) / vis_cols / layers
-    e_fr = np.abs(frame - rframe) / fr_cols / layers
-    e_head = np.abs(head - rhead) / np.maximum(n_text, 1)[:, None] / layers
-    e_aqf = np.abs(aqf - raqf) / layers
-    for name, e in (("tok", e_tok), ("frame", e_fr), ("head", e_head), ("aqf", e_aqf)):
+    frames = probe.n_vis // cfg.tokens_per_frame
+    e_tok = np.abs(tok - rtok)
+    e_fr = np.abs(frame - rframe)
+    e_head = np.abs(head - rhead) / np.maximum(np.abs(rhead), 1e-30)
+    e_head = np.where(np.abs(rhead) > 0, e_head, np.abs(head - rhead))
+    e_aqf = np.abs(aqf - raqf)
+    for name, e, bound in (("tok", e_tok, MAP_ABS), ("frame", e_fr, MAP_ABS), ("head (relative)", e_head, HEAD_REL),
+                           ("aqf", e_aqf, MAP_ABS)):
         if e.size:
             assert np.all(np.isfinite(e)), f"{label}: non-finite {name}"
-            assert e.max() <= MAP_ABS, f"{label}: {name} max abs {e.max():.3e}"
+            assert e.max() <= bound, f"{label}: {name} max error {e.max():.3e}"
     # planted frames: identical top-k on the head-summed frame map, per video
     off = 0
     for b, planted in enumerate(probe.planted):
@@ -101,4 +106,4 @@ def check_maps(gpu, ref, probe, layers=1, label=""):
             top_r = np.sort(np.argsort(-r, kind="stable")[:kk])
             np.testing.assert_array_equal(top_g, top_r, err_msg=f"{label}: top-k frames of video {b}")
         off += nf
-    return max(e.max() if e.size else 0 for e in (e_tok, e_fr, e_head, e_aqf))
+    return max(e.max() if e.size else 0 for e in (e_tok, e_fr, e_aqf))

@@ -100,7 +100,7 @@ def test_depth28_accumulated_evidence(cuda_lib):
             rows = _sample_rows(probe, per_video=24, seed=layer)
             _sampled_compare(cuda_lib, probe, rows, f"depth28 layer {layer}", out=out)
     torch.cuda.synchronize()
-    check_maps([np32(m) for m in maps], ref, probe, layers=cfg.layers, label="depth28 (sum of layers)")
+    check_maps([np32(m) for m in maps], ref, probe, label="depth28 (sum of layers)")
     ws.free()
 
 

@@ -78,7 +78,7 @@ def test_recompute_accumulates_over_layers(cuda_lib):
         maps = [out[k] for k in ("tok", "frame", "head", "aqf")]
         r = oracle_maps(probe)
         ref = r if ref is None else [a + b for a, b in zip(ref, r)]
-    check_maps([np32(m) for m in maps], ref, probe, layers=3, label="3 layers recompute")
+    check_maps([np32(m) for m in maps], ref, probe, label="3 layers recompute")
     ws.free()
 
 

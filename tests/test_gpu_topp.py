@@ -238,5 +238,5 @@ def test_coarse_evidence_matches_oracle(cuda_lib, name, block, tau):
     maps2 = cuda_lib.evisel_coarse_evidence(q, k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
                                             block, keep, ws, tok=maps[0].clone(), frame=maps[1].clone(),
                                             head=maps[2].clone(), aqf=maps[3].clone(), accumulate=True)
-    check_maps([np32(m) for m in maps2], [2 * w for w in want], probe, layers=2, label=f"{name} coarse x2")
+    check_maps([np32(m) for m in maps2], [2 * w for w in want], probe, label=f"{name} coarse x2")
     ws.free()
