@@ -32,22 +32,10 @@ def block_layout(n_vis: int, n_text: int, block: int):
     return out
 
 
-def round_bf16(x):
-    """Round float32 values to the nearest bfloat16 (ties to even), as float64."""
-    b = np.asarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
-    b = (b + 0x7FFF + ((b >> 16) & 1)) & 0xFFFF0000
-    return b.astype(np.uint32).view(np.float32).astype(np.float64)
-
-
-def block_means(k_video, n_vis: int, n_text: int, block: int, kbar_round=None):
-    """k_bar [n_blocks, Hkv, d] float64 for one video (Eq. 7). ``kbar_round``
-    "bf16": the mean taken in float32 and rounded to bfloat16, the precision in
-    which a bf16 tensor-core path takes its retention decision."""
+def block_means(k_video, n_vis: int, n_text: int, block: int):
+    """k_bar [n_blocks, Hkv, d] float64 for one video: the mean of each
+    block's keys (Eq. 7)."""
     k = np.asarray(k_video, dtype=np.float64)
-    if kbar_round == "bf16":
-        kf = np.asarray(k_video, dtype=np.float32)
-        return np.stack([round_bf16(kf[s:s + n].sum(axis=0, dtype=np.float32) / np.float32(n))
-                         for s, n in block_layout(n_vis, n_text, block)])
     return np.stack([k[s:s + n].mean(axis=0) for s, n in block_layout(n_vis, n_text, block)])
 
 
@@ -64,11 +52,11 @@ def select_prefix(p, tau):
     return sorted(keep)
 
 
-def retained_blocks(q, k, cu_seqlens, n_vis, block, tau_p, rows=None, heads=None, scale=None, kbar_round=None):
+def retained_blocks(q, k, cu_seqlens, n_vis, block, tau_p, rows=None, heads=None, scale=None):
     """S_i for the global token indices ``rows`` (default: all) and query heads
     ``heads`` (default: all). Returns a dict {(h, row): sorted list of the
     video's block ids}, and the matching p_i. as {(h, row): (block ids of H_i,
-    p over them)}. ``kbar_round``: see block_means."""
+    p over them)}."""
     q = np.asarray(q); k = np.asarray(k)
     n, hq, d = q.shape
     gq = hq // k.shape[1]
@@ -82,7 +70,7 @@ def retained_blocks(q, k, cu_seqlens, n_vis, block, tau_p, rows=None, heads=None
     for b in np.unique(video_of):
         s0, s1, nv = int(cu[b]), int(cu[b + 1]), int(n_vis[b])
         layout = block_layout(nv, s1 - s0 - nv, block)
-        kbar = block_means(k[s0:s1], nv, s1 - s0 - nv, block, kbar_round)
+        kbar = block_means(k[s0:s1], nv, s1 - s0 - nv, block)
         ends = np.array([s + ln for s, ln in layout])           # one past each block's last token
         for row in rows[video_of == b]:
             p_loc = int(row) - s0
@@ -187,14 +175,14 @@ def evidence_topp(q, k, cu_seqlens, n_vis, tokens_per_frame, block, kept, scale=
     return tok, frame, head, aqf
 
 
-def coarse_evidence(q, k, cu_seqlens, n_vis, tokens_per_frame, block, kept, scale=None, kbar_round=None):
+def coarse_evidence(q, k, cu_seqlens, n_vis, tokens_per_frame, block, kept, scale=None):
     """Evidence maps from the coarse token-level map (Appendix Eq. 10-11): for a
     text row i, a_im = q_i k_m / sqrt(d) for the keys m of its own block up to
     i (E_i; there is no system prefix here), a_im = g_ij for the tokens of each
     retained block K_j in S_i = ``kept[(h, row)]``, -inf elsewhere; the map is
     the row softmax of a. Its mass on the visual tokens is summed over the
     text rows into tok [Hq, sum n_vis], then frame, head and aqf as in the
-    exact evidence (Sec. 3.2). ``kbar_round``: see block_means."""
+    exact evidence (Sec. 3.2)."""
     q = np.asarray(q); k = np.asarray(k)
     n, hq, d = q.shape
     gq = hq // k.shape[1]
@@ -213,7 +201,7 @@ def coarse_evidence(q, k, cu_seqlens, n_vis, tokens_per_frame, block, kept, scal
         s0, s1, nv = int(cu[b]), int(cu[b + 1]), int(n_vis[b])
         n_text = s1 - s0 - nv
         layout = block_layout(nv, n_text, block)
-        kbar = block_means(k[s0:s1], nv, n_text, block, kbar_round)
+        kbar = block_means(k[s0:s1], nv, n_text, block)
         for h in range(hq):
             t_map = np.zeros(nv)
             for row in range(s0 + nv, s1):

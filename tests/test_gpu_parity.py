@@ -63,12 +63,51 @@ def test_single_full(cuda_lib):
     _full_compare(cuda_lib, wl.make_probe(wl.CONFIGS["single"]), "single")
 
 
+def _whole_tiles(probe):
+    """{label: global rows} of whole query tiles that, over all heads, run every
+    item class of the attention kernel: the visual row tile with the most kept
+    kv tiles (the longest items), the first visual tile, the last visual tile
+    of each video (ragged where n_vis is not a multiple of the tile), and every
+    text row of each video (its kv range is split over several items whose
+    partials the combine merges). All heads of a tile cover both the two-slot
+    items and the one-slot item of a KV group's odd last head."""
+    T = probe.cfg.tile
+    counts = np.diff(probe.row_ptr)
+    tiles = {}
+    r0 = 0
+    best = (-1, None)
+    for b in range(len(probe.n_vis)):
+        s0, s1, nv = int(probe.cu_seqlens[b]), int(probe.cu_seqlens[b + 1]), int(probe.n_vis[b])
+        n_vt = -(-nv // T)
+        for t in range(n_vt):
+            if counts[r0 + t] > best[0]:
+                best = (int(counts[r0 + t]), (b, t))
+        if n_vt and b == 0:
+            tiles[f"video {b} first visual tile"] = np.arange(s0, s0 + min(T, nv))
+        if n_vt:
+            tiles[f"video {b} last visual tile ({nv - (n_vt - 1) * T} rows)"] = np.arange(s0 + (n_vt - 1) * T, s0 + nv)
+        if s1 > s0 + nv:
+            tiles[f"video {b} text rows ({s1 - s0 - nv})"] = np.arange(s0 + nv, s1)
+        r0 += n_vt
+    if best[1] is not None:
+        b, t = best[1]
+        s0, nv = int(probe.cu_seqlens[b]), int(probe.n_vis[b])
+        tiles[f"video {b} visual tile {t} ({best[0]} kv tiles)"] = np.arange(s0 + t * T, s0 + min((t + 1) * T, nv))
+    return tiles
+
+
+def _tile_compare(probe, out, label):
+    for name, rows in _whole_tiles(probe).items():
+        _sampled_compare(None, probe, rows, f"{label}: {name}", out=out)
+
+
 def test_long65k_sampled_and_maps(cuda_lib):
     probe = wl.make_probe(wl.CONFIGS["long65k"])
     out, ws = run_cuda(cuda_lib, probe)
     ws.free()
     rows = _sample_rows(probe, per_video=96)
     _sampled_compare(cuda_lib, probe, rows, "long65k", out=out)
+    _tile_compare(probe, out, "long65k")
     check_maps([np32(out[k]) for k in ("tok", "frame", "head", "aqf")], oracle_maps(probe), probe,
                label="long65k")
 
@@ -79,6 +118,7 @@ def test_varlen8_sampled_and_maps(cuda_lib):
     ws.free()
     rows = _sample_rows(probe, per_video=16)
     _sampled_compare(cuda_lib, probe, rows, "varlen8", out=out)
+    _tile_compare(probe, out, "varlen8")
     check_maps([np32(out[k]) for k in ("tok", "frame", "head", "aqf")], oracle_maps(probe), probe,
                label="varlen8")
 

@@ -1,16 +1,21 @@
 """GPU parity of the top-p block retention (evisel_topp_mask) against
-oracle.topp.retained_blocks, through the C ABI.
+oracle.topp.retained_blocks (float64 block means and logits, Eq. 7-9),
+through the C ABI.
 
-Several sets can be "the" answer only at ties, so each GPU set is checked
-against the oracle's p (block means rounded to bf16 as the tensor-core path
-takes them): it holds the row's own block and blocks of H_i only; its mass
-reaches tau_p; it is minimal (without its least block the mass is below
-tau_p); and it is a top set (no dropped block has a larger p). Each check
-allows EPS of p: the GPU's logits are fp32 sums of bf16 products, and its
-order resolves logits to (max - min) / 16384 over H_i.
-The tile union is checked bit for bit against the union of the GPU's own
-sets, and, read as a mask, it drives the probe, whose rows match the oracle.
+Several sets are correct where block logits (nearly) tie, so each GPU set is
+checked against the oracle's p with the retention rule's four properties: it
+holds the row's own block and blocks of H_i only; its mass reaches tau_p; it is
+minimal (without its least block the mass is below tau_p); and it is a top set
+(no dropped block has a larger p). Each property is allowed the error of the
+GPU's logits, bounded per block from its arithmetic (_logit_bounds): the block
+mean summed in fp32 and rounded to bf16 (the tensor cores' operand type), the
+q . k_bar products accumulated in fp32, and the fp32 scaling; and the error of
+its fp32 mass sums. The tile union is checked bit for bit against the union of
+the GPU's own sets, and, read as a mask, it drives the probe, whose rows match
+the oracle.
 """
+import math
+
 import numpy as np
 import pytest
 
@@ -21,8 +26,52 @@ from gpu_helpers import check_lse, check_o, to_device
 
 pytestmark = pytest.mark.gpu
 
-EPS = 2e-5
-LOG2_EPS = 3e-5      # fp32 logits (bf16 products) against the oracle's float64, in log2 units
+U32 = 2.0 ** -24     # fp32 unit roundoff
+U16 = 2.0 ** -9      # bf16 unit roundoff (round to nearest even)
+
+
+def _logit_bounds(q, k, cu, n_vis, block, rows):
+    """{(h, row): eps over the row's H_i}: a bound on |g_gpu - g| (natural-log
+    units) for every block of H_i, from the builder's arithmetic:
+      k_bar32 = fp32 sum of the block's n bf16 keys / n:
+                |k_bar32 - k_bar| <= n U32 mean|k|                     (a)
+      k~      = bf16(k_bar32): |k~ - k_bar32| <= U16 |k_bar32|          (b)
+      S       = sum_d q_d k~_d, bf16 products exact in fp32, accumulated in
+                fp32 (one rounding of at most 2 U32 per addition, whatever
+                the order): |S - q.k~| <= 2 d U32 sum_d |q_d k~_d|       (c)
+      x       = S scale log2(e) in fp32, then u = max - x: a few roundings of
+                at most U32 relative to the row's largest |g|            (d)
+    so eps_j = scale (sum_d |q_d| delta_jd + 2 d U32 sum_d |q_d| (|k_bar_jd|
+    + delta_jd)) + 8 U32 max_j |g_j|, with delta_jd = (a) + U16 (|k_bar_jd| + (a))."""
+    q = np.asarray(q, np.float64)
+    k = np.asarray(k, np.float64)
+    n, hq, d = q.shape
+    gq = hq // k.shape[1]
+    scale = 1.0 / math.sqrt(d)
+    cu = np.asarray(cu)
+    out = {}
+    for row in rows:
+        b = int(np.searchsorted(cu, row, side="right") - 1)
+        s0, s1, nv = int(cu[b]), int(cu[b + 1]), int(n_vis[b])
+        layout = oracle.block_layout(nv, s1 - s0 - nv, block)
+        ends = np.array([s + ln for s, ln in layout])
+        hist = np.nonzero(ends <= row - s0)[0]
+        if hist.size == 0:
+            for h in range(hq):
+                out[(h, int(row))] = np.zeros(0)
+            continue
+        kv = k[s0:s1]
+        kbar = np.stack([kv[layout[j][0]:layout[j][0] + layout[j][1]].mean(axis=0) for j in hist])
+        mabs = np.stack([np.abs(kv[layout[j][0]:layout[j][0] + layout[j][1]]).mean(axis=0) for j in hist])
+        lens = np.array([layout[j][1] for j in hist], np.float64)[:, None, None]
+        a = lens * U32 * mabs
+        delta = a + U16 * (np.abs(kbar) + a)
+        for h in range(hq):
+            qa = np.abs(q[row, h])
+            g = scale * (kbar[:, h // gq] @ q[row, h])
+            eps = scale * (delta[:, h // gq] @ qa + 2 * d * U32 * ((np.abs(kbar[:, h // gq]) + delta[:, h // gq]) @ qa))
+            out[(h, int(row))] = eps + 8 * U32 * np.abs(g).max()
+    return out
 
 
 def _gpu_sets(ev, probe, block, tau, rows):
@@ -43,10 +92,16 @@ def _gpu_sets(ev, probe, block, tau, rows):
     return sets, keep, uni
 
 
-def _check_sets(gpu, probs, cu, n_vis, block, tau, label):
+def _check_sets(gpu, probs, bounds, cu, n_vis, block, tau, label):
+    """The retention rule's properties, each allowed the logit bound eps of
+    the blocks involved: a logit off by at most e moves p by a factor within
+    exp(+-2 e_max), and the builder's fp32 sums of 2^x over |H_i| blocks (x
+    with ex2.approx, relative error below 2^-21) add at most eta of mass."""
     cu = np.asarray(cu)
+    worst = -math.inf
     for (h, row), ids in gpu.items():
         hist, p = probs[(h, row)]
+        eps = bounds[(h, row)]
         b = int(np.searchsorted(cu, row, side="right") - 1)
         pos = row - int(cu[b])
         nv = int(n_vis[b])
@@ -59,13 +114,20 @@ def _check_sets(gpu, probs, cu, n_vis, block, tau, label):
             continue
         kept = np.isin(hist, s)
         mass = p[kept].sum()
-        assert mass >= tau - EPS, (label, h, row, "mass", mass)
-        assert mass - p[kept].min() < tau + EPS, (label, h, row, "not minimal", mass, p[kept].min())
+        e_max = float(eps.max())
+        eta = 2.0 ** -21 + (hist.size + 2) * 2 * U32
+        lo = tau * math.exp(-2 * e_max) - eta
+        hi = tau * math.exp(2 * e_max) + eta + 2 * e_max
+        assert mass >= lo, (label, h, row, "mass", mass, lo)
+        assert mass - p[kept].min() < hi, (label, h, row, "not minimal", mass, p[kept].min(), hi)
         if (~kept).any():
-            # top set, up to the builder's resolution: log2 p within (max - min) / 16384 of each other may tie
-            lp = np.log2(p[p > 0])
-            res = (lp.max() - lp.min()) / 16384 + LOG2_EPS
-            assert np.log2(p[kept].min()) >= np.log2(p[~kept].max()) - res, (label, h, row, "not a top set")
+            # top set: every kept block's logit, raised by its bound, reaches every
+            # dropped block's logit lowered by its own (log p differs from g by a constant)
+            with np.errstate(divide="ignore"):
+                lp = np.log(p)
+            worst = max(worst, float(np.max(lp[~kept] - eps[~kept]) - np.min(lp[kept] + eps[kept])))
+            assert np.min(lp[kept] + eps[kept]) >= np.max(lp[~kept] - eps[~kept]), (label, h, row, "not a top set")
+    return worst
 
 
 def _all_rows(probe):
@@ -77,9 +139,9 @@ def test_topp_sets_small(cuda_lib, name, block, tau):
     probe = wl.make_probe(wl.CONFIGS[name])
     rows = _all_rows(probe)
     gpu, _, _ = _gpu_sets(cuda_lib, probe, block, tau, rows)
-    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, tau, rows=rows,
-                                      kbar_round="bf16")
-    _check_sets(gpu, probs, probe.cu_seqlens, probe.n_vis, block, tau, name)
+    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, tau, rows=rows)
+    bounds = _logit_bounds(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, rows)
+    _check_sets(gpu, probs, bounds, probe.cu_seqlens, probe.n_vis, block, tau, name)
 
 
 @pytest.mark.parametrize("name,block,n_rows", [("long65k", 64, 24), ("varlen8", 16, 24)])
@@ -89,9 +151,9 @@ def test_topp_sets_sampled(cuda_lib, name, block, n_rows):
     n = int(probe.cu_seqlens[-1])
     rows = np.unique(np.concatenate([[0, n - 1], probe.cu_seqlens[1:-1], rng.integers(0, n, n_rows)]))
     gpu, _, _ = _gpu_sets(cuda_lib, probe, block, 0.97, rows)
-    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, 0.97, rows=rows,
-                                      kbar_round="bf16")
-    _check_sets(gpu, probs, probe.cu_seqlens, probe.n_vis, block, 0.97, name)
+    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, 0.97, rows=rows)
+    bounds = _logit_bounds(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, rows)
+    _check_sets(gpu, probs, bounds, probe.cu_seqlens, probe.n_vis, block, 0.97, name)
 
 
 EDGE = {
@@ -109,9 +171,9 @@ def test_topp_edge_cases(cuda_lib, name, block, tau):
     probe = _custom(**EDGE[name])
     rows = _all_rows(probe)
     gpu, _, _ = _gpu_sets(cuda_lib, probe, block, tau, rows)
-    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, tau, rows=rows,
-                                      kbar_round="bf16")
-    _check_sets(gpu, probs, probe.cu_seqlens, probe.n_vis, block, min(tau, 1.0 - 1e-6), name)
+    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, tau, rows=rows)
+    bounds = _logit_bounds(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, rows)
+    _check_sets(gpu, probs, bounds, probe.cu_seqlens, probe.n_vis, block, min(tau, 1.0 - 1e-6), name)
 
 
 def test_topp_union_drives_the_probe(cuda_lib):
@@ -215,7 +277,8 @@ def test_keep_refused_where_it_does_not_apply(cuda_lib):
 @pytest.mark.parametrize("name,block,tau", [("single", 16, 0.5), ("tiny", 16, 0.9)])
 def test_coarse_evidence_matches_oracle(cuda_lib, name, block, tau):
     """Evidence of the coarse map (Eq. 10-11) on the GPU's own retained sets
-    against the oracle taken with the same sets and bf16 block means."""
+    against the oracle taken with the same sets and float64 block means (Eq. 7),
+    at the maps' tolerances."""
     import torch
     from gpu_helpers import check_maps, np32
     probe = wl.make_probe(wl.CONFIGS[name])
@@ -231,8 +294,7 @@ def test_coarse_evidence_matches_oracle(cuda_lib, name, block, tau):
     text_rows = np.concatenate([np.arange(int(probe.cu_seqlens[b]) + int(probe.n_vis[b]), int(probe.cu_seqlens[b + 1]))
                                 for b in range(len(probe.n_vis))])
     kept = _sets_from_keep(keep, text_rows, probe.cu_seqlens, probe.n_vis, block)
-    want = oracle.coarse_evidence(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, block, kept,
-                                  kbar_round="bf16")
+    want = oracle.coarse_evidence(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, block, kept)
     check_maps([np32(m) for m in maps], list(want), probe, label=f"{name} coarse evidence")
     # accumulate: a second call adds the same maps
     maps2 = cuda_lib.evisel_coarse_evidence(q, k, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,

@@ -724,15 +724,6 @@ def test_H3_catches_an_ascending_order(monkeypatch):
         test_H3_topp_planted_block_takes_the_mass()
 
 
-def test_H6_round_bf16_matches_torch():
-    torch = pytest.importorskip("torch")
-    rng = np.random.default_rng(47)
-    x = np.concatenate([rng.standard_normal(4096).astype(np.float32) * 10 ** rng.uniform(-6, 6, 4096),
-                        np.array([1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -(1.0 + 2 ** -8)], np.float32)])
-    from oracle.topp import round_bf16
-    np.testing.assert_array_equal(round_bf16(x), torch.from_numpy(x).to(torch.bfloat16).double().numpy())
-
-
 def test_H7_evidence_with_every_block_kept_is_the_dense_evidence():
     c = _topp_case(48, videos=((16, 6), (12, 5)))
     sets, _ = oracle.retained_blocks(c["q"], c["k"], c["cu"], c["n_vis"], 4, 1.0 - 1e-12)
@@ -796,8 +787,8 @@ def test_C2_catches_block_sums_for_means(monkeypatch):
     import oracle.topp as ot
     good = ot.block_means
 
-    def sums(k_video, n_vis, n_text, block, kbar_round=None):
-        m = good(k_video, n_vis, n_text, block, kbar_round)
+    def sums(k_video, n_vis, n_text, block):
+        m = good(k_video, n_vis, n_text, block)
         lens = np.array([ln for _, ln in ot.block_layout(n_vis, n_text, block)], np.float64)
         return m * lens[:, None, None]
     monkeypatch.setattr(ot, "block_means", sums)
