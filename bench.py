@@ -2,11 +2,16 @@
 
 One step = the whole hot path on one batch: evisel_probe_attention (block-sparse
 GQA attention + split-KV merge, text-logit spill) and evisel_evidence_reduce
-(token / frame / head maps and A_qf). Default workload: the 65,664-token probe
-(1024 frames x 64 pooled tokens + 128 text tokens, 28 query / 4 KV heads,
+(token / frame / head maps and A_qf). The headline workload is the 65,664-token
+probe (1024 frames x 64 pooled tokens + 128 text tokens, 28 query / 4 KV heads,
 d = 128, 128-token tiles, sink + 16-tile window + 32 random tiles per visual
 row tile). Inputs are synthetic (seeded), resident in HBM when the timed region
 starts, and larger than L2, so no flush is needed between steps.
+
+The same line carries, under "configs", the step timed the same way on every
+workload: the 544-token and 4,160-token probes (L2 flushed before every step),
+the 28-layer probe (one step = the probe and the accumulating evidence pass of
+all 28 layers, each with its own Q/K/V) and the 8-video packed batch.
 
 Prints one JSON line (rank 0). --impl reference times the float64 oracle on
 the host cores instead (bounded sample of the same workload).
@@ -22,6 +27,7 @@ import subprocess
 import sys
 import tempfile
 import time
+from concurrent.futures import ThreadPoolExecutor
 
 import numpy as np
 
@@ -248,6 +254,183 @@ def _config_dict(cfg, st):
             "l2": "inputs larger than L2 (no flush)", "parallelism": "replicas"}
 
 
+L2_FLUSH_BYTES = 256 * 1024 * 1024     # twice the GB300's L2
+
+
+def _gpu_local_cpus(device_index):
+    """Host CPUs on the NUMA node of the GPU's PCI device (empty if unknown):
+    pinned host buffers first touched from these CPUs sit in the memory
+    nearest to the GPU, and copies from them take the shortest path."""
+    import torch
+    try:
+        p = torch.cuda.get_device_properties(device_index)
+        bus = f"{p.pci_domain_id:04x}:{p.pci_bus_id:02x}:{p.pci_device_id:02x}.0"
+        with open(f"/sys/bus/pci/devices/{bus}/local_cpulist") as fh:
+            spec = fh.read().strip()
+    except (AttributeError, OSError, ValueError):
+        return set()
+    cpus = set()
+    for part in spec.split(","):
+        if part:
+            a, _, b = part.partition("-")
+            cpus |= set(range(int(a), int(b or a) + 1))
+    return cpus & os.sched_getaffinity(0)
+
+
+def bench_config(ev, name, args, peaks):
+    """The step (probe + evidence over every layer) of one workload, timed on
+    the launch stream with CUDA events: the whole step, and per layer the
+    probe call and the evidence call. Workloads whose inputs fit in L2 get a
+    256 MB write before every timed step (outside the timed interval)."""
+    import torch
+    cfg = wl.CONFIGS[name]
+    layers = cfg.layers
+    if layers > 1:
+        mask = wl.build_mask(cfg)
+        with ThreadPoolExecutor(max(1, min(8, os.cpu_count() or 1))) as ex:
+            probes = list(ex.map(lambda l: wl.make_probe(cfg, l, mask=mask), range(layers)))
+    else:
+        probes = [wl.make_probe(cfg)]
+    probe = probes[0]
+    st = workload_stats(probe)                  # per layer: every layer has the same shapes and mask
+    dev = []
+    for p in probes:
+        dev.append(tuple(torch.from_numpy(x).cuda().to(torch.bfloat16) for x in (p.q, p.k, p.v)))
+    del probes
+    q0 = dev[0][0]
+    n, hq, d = q0.shape
+    in_bytes = layers * sum(t.numel() * t.element_size() for t in dev[0])
+    flush = in_bytes + st["spill_bytes"] < 4 * L2_FLUSH_BYTES
+    flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda") if flush else None
+    o = torch.empty_like(q0)
+    lse = torch.empty((hq, n), dtype=torch.float32, device="cuda")
+    total_vis = int(np.sum(probe.n_vis))
+    frames = total_vis // cfg.tokens_per_frame
+    maps = [torch.zeros((hq, total_vis), device="cuda"), torch.zeros((hq, frames), device="cuda"),
+            torch.zeros((len(probe.n_vis), hq), device="cuda"), torch.zeros((frames,), device="cuda")]
+    ws = ev.Workspace()
+    stream = torch.cuda.current_stream()
+
+    def step(marks=None):
+        for layer, (q, k, v) in enumerate(dev):
+            if marks:
+                marks[layer][0].record(stream)
+            ev.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                      probe.row_ptr, probe.col_idx, ws=ws, o=o, lse=lse)
+            if marks:
+                marks[layer][1].record(stream)
+            ev.evisel_evidence_reduce(ws, hq, probe.n_vis, cfg.tokens_per_frame, len(probe.n_vis), tok=maps[0],
+                                      frame=maps[1], head=maps[2], aqf=maps[3], accumulate=layer > 0)
+            if marks:
+                marks[layer][2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if ev.evisel_status(ws) != 0:
+        raise RuntimeError(f"{name}: device status reported an error")
+    ev_t = lambda: torch.cuda.Event(enable_timing=True)
+    bounds = [(ev_t(), ev_t()) for _ in range(args.steps)]
+    marks = [[[ev_t() for _ in range(3)] for _ in range(layers)] for _ in range(args.steps)]
+    for i in range(args.steps):
+        if flush_buf is not None:
+            flush_buf.zero_()
+        bounds[i][0].record(stream)
+        step(marks[i])
+        bounds[i][1].record(stream)
+    torch.cuda.synchronize()
+    status = ev.evisel_status(ws)
+    ws.free()
+    if status != 0:
+        raise RuntimeError(f"{name}: device status reported an error")
+    if not all(bool(torch.isfinite(m).all()) for m in maps):
+        raise RuntimeError(f"{name}: non-finite evidence maps")
+    step_ms = sum(a.elapsed_time(b) for a, b in bounds) / args.steps
+    attn_ms = sum(m[0].elapsed_time(m[1]) for s_ in marks for m in s_) / args.steps
+    ev_ms = sum(m[1].elapsed_time(m[2]) for s_ in marks for m in s_) / args.steps
+    flop = layers * st["flop"]
+    attn_tflops = flop / (attn_ms * 1e-3) / 1e12
+    ev_gbs = layers * st["evidence_bytes"] / (ev_ms * 1e-3) / 1e9
+    return {"workload": f"{cfg.name}: {cfg.description}", "tokens": st["n_tok"], "layers": layers,
+            "videos": cfg.num_videos, "kept_tiles_per_layer": st["tiles"], "flop_per_step": flop,
+            "step_ms": step_ms, "tflops": flop / (step_ms * 1e-3) / 1e12,
+            "tokens_per_s": st["n_tok"] * layers / (step_ms * 1e-3),
+            "attention_ms": attn_ms, "attention_tflops": attn_tflops,
+            "attention_frac_of_bf16_peak": attn_tflops / peaks["bf16"],
+            "attention_ms_at_60pct_of_peak": flop / (0.6 * peaks["bf16"] * 1e12) * 1e3,
+            "evidence_ms": ev_ms, "evidence_bytes": layers * st["evidence_bytes"], "evidence_gbs": ev_gbs,
+            "evidence_frac_of_hbm": ev_gbs / peaks["hbm"],
+            "l2": "256 MB write before every step (untimed)" if flush else "inputs larger than L2 (no flush)"}
+
+
+def bench_topp_sparse(ev, args, peaks):
+    """The top-p path (Appendix Eq. 6-9, blocks of N_v tokens, tau_p = 0.97)
+    where retention keeps a small share of each row's history: the 65K probe
+    with concentrated attention (long65k_sparse). Times the builder, the probe
+    on the tile union with the per-row bits, and, for comparison, the probe on
+    the same inputs under the static mask; the kept share is counted on a
+    sample of rows from the builder's own bits."""
+    import torch
+    cfg = wl.CONFIGS["long65k_sparse"]
+    probe = wl.make_probe(cfg)
+    st = workload_stats(probe)
+    q, k, v = (torch.from_numpy(x).cuda().to(torch.bfloat16) for x in (probe.q, probe.k, probe.v))
+    n, hq, d = q.shape
+    npf, tau = cfg.tokens_per_frame, 0.97
+    o = torch.empty_like(q)
+    lse = torch.empty((hq, n), dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(fn):
+        for _ in range(max(1, args.warmup)):
+            fn()
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(args.steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / args.steps
+
+    ws = ev.Workspace()
+    keep, uni, ws = ev.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, npf, tau, ws=ws)
+    build_ms = timed(lambda: ev.evisel_topp_mask(q, k, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, npf, tau,
+                                                 ws=ws))
+    row_ptr, col_idx = ev.tile_union_to_csr(uni, probe.n_vis, cfg.tile)
+    uargs = (q, k, v, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, row_ptr, col_idx)
+    ws_p = ev.Workspace()
+    union_ms = timed(lambda: ev.evisel_probe_attention(*uargs, ws=ws_p, o=o, lse=lse, keep=keep, keep_block=npf))
+    sargs = (q, k, v, probe.cu_seqlens, probe.n_vis, npf, cfg.tile, probe.row_ptr, probe.col_idx)
+    ws_s = ev.Workspace()
+    static_ms = timed(lambda: ev.evisel_probe_attention(*sargs, ws=ws_s, o=o, lse=lse))
+    status = [ev.evisel_status(w) for w in (ws, ws_p, ws_s)]
+    # kept share on sampled rows: retained blocks (own block excluded) over |H_i|
+    rows = np.random.default_rng(0).integers(0, n, 256)
+    bits = keep[:, :, torch.as_tensor(rows, device="cuda")].cpu().numpy().view(np.uint32)   # [hq, words, rows]
+    bits = np.ascontiguousarray(bits.transpose(0, 2, 1))                                       # [hq, rows, words]
+    kept = np.unpackbits(bits.view(np.uint8), axis=2).sum(axis=2).astype(np.int64) - 1         # own block excluded
+    nv = int(probe.n_vis[0])
+    hist = np.where(rows < nv, rows // npf, nv // npf + (rows - nv) // npf)
+    share = (kept / np.maximum(hist, 1)[None, :])[:, hist >= 64]
+    for w in (ws, ws_p, ws_s):
+        w.free()
+    if any(status):
+        raise RuntimeError("device status reported an error")
+    # union work in the attention's convention: every kept (row tile, kv tile) pair, full tiles, plus text rows
+    ust = workload_stats(wl.Probe(cfg, 0, probe.q[:0], probe.k[:0], probe.v[:0], probe.cu_seqlens, probe.n_vis,
+                                  row_ptr, col_idx, probe.planted))
+    return {"workload": f"{cfg.name}: {cfg.description}", "block": npf, "tau_p": tau,
+            "builder_ms": build_ms,
+            "kept_share_of_history": {"median": float(np.median(share)), "mean": float(np.mean(share)),
+                                      "sampled_rows": int(share.shape[1]), "heads": hq},
+            "union_tiles": int(row_ptr[-1]), "static_mask_tiles": int(probe.row_ptr[-1]),
+            "probe_on_union_ms": union_ms, "probe_on_union_tflops": ust["flop"] / (union_ms * 1e-3) / 1e12,
+            "probe_on_union_frac_of_bf16_peak": ust["flop"] / (union_ms * 1e-3) / 1e12 / peaks["bf16"],
+            "probe_static_mask_ms": static_ms,
+            "builder_plus_union_probe_ms": build_ms + union_ms}
+
+
 def bench_ours(args, cfg):
     import torch
     import torch.distributed as dist
@@ -327,6 +510,11 @@ def bench_ours(args, cfg):
     # on a second stream into a second set of device buffers, so that the inputs
     # of step i + 1 and the maps of step i move while step i computes (the
     # first step's inputs and the last step's maps are inside the timed region).
+    # Host buffers on the GPU's NUMA node: the process runs on the GPU's local
+    # CPUs from here on, so that the pinned buffers are first touched there.
+    local_cpus = _gpu_local_cpus(local)
+    if local_cpus:
+        os.sched_setaffinity(0, local_cpus)
     hq_, hk_, hv_ = (t.cpu().pin_memory() for t in (q, k, v))
     host_maps = [m.cpu().pin_memory() for m in maps]
     h2d = sum(t.numel() * t.element_size() for t in (hq_, hk_, hv_))
@@ -385,6 +573,33 @@ def bench_ours(args, cfg):
     # the copies are done: the last step's maps are on the host
     if not all(np.isfinite(hm.numpy()).all() for hm in host_maps):
         raise RuntimeError("non-finite evidence maps")
+
+    # The copies alone, on the copy stream: what bounds the pipelined loop
+    # when they take longer than the step.
+    def copy_ms(fn):
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        c0.record(copy_stream)
+        for _ in range(args.steps):
+            fn()
+        c1.record(copy_stream)
+        torch.cuda.synchronize()
+        return c0.elapsed_time(c1) / args.steps
+
+    def h2d_only():
+        with torch.cuda.stream(copy_stream):
+            for dst, src in zip(bufs[1], (hq_, hk_, hv_)):
+                dst.copy_(src, non_blocking=True)
+
+    def d2h_only():
+        with torch.cuda.stream(copy_stream):
+            for hm, m in zip(host_maps, map_bufs[1]):
+                hm.copy_(m, non_blocking=True)
+
+    h2d_ms = copy_ms(h2d_only)
+    d2h_ms = copy_ms(d2h_only)
     del bufs[1], map_bufs[1]
 
     # The intra-frame cue A_if (a row beyond the probe step), timed on its own
@@ -519,6 +734,29 @@ def bench_ours(args, cfg):
     if status != 0:
         raise RuntimeError("device status reported an error")
 
+    topp_sparse = None if args.no_configs else bench_topp_sparse(ev, args, peaks)
+    torch.cuda.empty_cache()
+
+    # Every workload's step, timed the same way (replicas: each rank times its own).
+    configs = {}
+    if not args.no_configs:
+        cclk = ClockSampler(local)
+        cclk.start()
+        for name in ("tiny", "single", "depth28", "varlen8"):
+            configs[name] = bench_config(ev, name, args, peaks)
+            torch.cuda.empty_cache()
+        configs["clocks"] = cclk.stop()
+    configs["long65k"] = {"workload": f"{cfg.name}: {cfg.description}", "tokens": st["n_tok"], "layers": 1,
+                          "videos": cfg.num_videos, "kept_tiles_per_layer": st["tiles"], "flop_per_step": st["flop"],
+                          "step_ms": ms_step, "tflops": st["flop"] / (ms_step * 1e-3) / 1e12,
+                          "tokens_per_s": st["n_tok"] / (ms_step * 1e-3),
+                          "attention_ms": attn_avg, "attention_tflops": attn_tflops,
+                          "attention_frac_of_bf16_peak": attn_tflops / peaks["bf16"],
+                          "attention_ms_at_60pct_of_peak": st["flop"] / (0.6 * peaks["bf16"] * 1e12) * 1e3,
+                          "evidence_ms": ev_avg, "evidence_bytes": st["evidence_bytes"], "evidence_gbs": ev_gbs,
+                          "evidence_frac_of_hbm": ev_gbs / peaks["hbm"], "l2": "inputs larger than L2 (no flush)",
+                          "note": "the headline step (value, attention, evidence above)"}
+
     line = None
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
@@ -552,9 +790,17 @@ def bench_ours(args, cfg):
                                 "ms": cf_ms, "gbs": cf_bytes / (cf_ms * 1e-3) / 1e9,
                                 "frac_of_hbm": cf_bytes / (cf_ms * 1e-3) / 1e9 / peaks["hbm"], "bytes": cf_bytes},
                 "e2e": {"value": _whole_job_tflops(world, st["flop"], e2e_ms), "unit": "TFLOP/s",
-                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+                        "h2d_ms_alone": h2d_ms, "h2d_gbs": h2d / (h2d_ms * 1e-3) / 1e9,
+                        "d2h_ms_alone": d2h_ms, "d2h_gbs": d2h / (d2h_ms * 1e-3) / 1e9,
+                        "host_buffers": (f"pinned, first touched on the GPU's {len(local_cpus)} local CPUs"
+                                         if local_cpus else "pinned (GPU NUMA node unknown)"),
+                        "pipeline": "inputs of step i+1 and maps of step i copied on a second stream while "
+                                    "step i computes"},
                 "gpu_launches": args.steps * (4 if _has_combine(probe) else 3),
-                "clocks": clk}
+                "clocks": clk,
+                "topp_sparse": topp_sparse,
+                "configs": configs}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         flop, dt, nrows = run_oracle(probe, args.ref_rows)
         line["cpu_baseline"] = {"value": flop / dt / 1e12, "unit": "TFLOP/s", "cores": os.cpu_count(),
@@ -587,9 +833,12 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", default="long65k", choices=sorted(wl.CONFIGS))
+    ap.add_argument("--config", default="long65k", choices=sorted(n for n, c in wl.CONFIGS.items() if c.layers == 1),
+                    help="workload of the headline step (single-layer workloads; the 28-layer step is "
+                         "timed under 'configs')")
     ap.add_argument("--ref-rows", type=int, default=256)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true", help="skip the per-workload steps under 'configs'")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

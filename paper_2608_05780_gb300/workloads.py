@@ -77,6 +77,8 @@ class ProbeConfig:
     qkv_seed: object = None   # seed for Q/K/V draws (default: ``seed``)
     scale_inputs: bool = True  # Q/K/V ~ N(0,1)/sqrt(d); False gives "sharp" N(0,1)
     description: str = ""
+    # "clustered": concentrated attention (see _clustered); default: i.i.d. draws
+    regime: str = "iid"
 
     @property
     def n_vis(self):
@@ -129,6 +131,11 @@ CONFIGS = {
         plant=_plant_count(0.02, (384,)), seed=3, mask_seed=3,
         description="profiling-size variant of long65k: 384 frames x 64 tokens + 128 text (24,704 tokens); "
                     "same heads, tiles and mask recipe; inputs still larger than L2"),
+    "long65k_sparse": ProbeConfig(
+        "long65k_sparse", (1024,), 64, (128,), 28, 4, 128, 128, 16, extra=32, seed=5, mask_seed=3,
+        scale_inputs=False, regime="clustered",
+        description="long65k's shapes with concentrated attention (clustered keys and queries, see "
+                    "_clustered): the regime where top-p retention keeps a small share of each row's history"),
     "varlen8": ProbeConfig(
         "varlen8", _C5_FRAMES, 16, _C5_TEXT, 28, 4, 128, 128, 8,
         plant=_plant_count(0.05, _C5_FRAMES), seed=4, qkv_seed=(4, 1),
@@ -192,6 +199,52 @@ def _planted_frames(cfg: ProbeConfig):
     return out
 
 
+CLUSTER_KEY_WEIGHT = 3.0      # alpha: weight of a block's topic in its keys
+CLUSTER_QUERY_NOISE = 0.25    # gamma: weight of a query's own noise
+CLUSTER_RECENT = 4            # targets of a row tile: its most recent earlier blocks ...
+CLUSTER_RANDOM = 4            # ... and this many random earlier blocks
+
+
+def _clustered(cfg: ProbeConfig, q, k, cu, rng):
+    """Concentrated attention (a stand-in for the regime where top-p retention
+    keeps few blocks): every block of N_v tokens of a video has a topic vector
+    c_j ~ N(0, I_d) per KV group, and its keys are alpha c_j + N(0, I_d); every
+    query row tile (tiles of ``cfg.tile`` rows over the visual rows, then over
+    the text rows) draws target blocks among the blocks that end before it (its
+    CLUSTER_RECENT most recent ones and CLUSTER_RANDOM random earlier ones),
+    and its queries are s + gamma N(0, I_d) with s the targets' topics summed
+    and divided by sqrt(#targets) (per KV group, shared by the group's heads).
+    ``q`` and ``k`` hold the N(0, 1) draws on entry and are overwritten."""
+    d, npf, T = cfg.head_dim, cfg.tokens_per_frame, cfg.tile
+    gq = cfg.hq // cfg.hkv
+    for b in range(cfg.num_videos):
+        s0, nv, nt = int(cu[b]), cfg.n_vis[b], cfg.n_text[b]
+        n_blk = nv // npf + -(-nt // npf)
+        topic = rng.standard_normal((n_blk, cfg.hkv, d), dtype=np.float32)
+        blk_of = np.concatenate([np.arange(nv) // npf, nv // npf + np.arange(nt) // npf])
+        k[s0:s0 + nv + nt] = np.float32(CLUSTER_KEY_WEIGHT) * topic[blk_of] + k[s0:s0 + nv + nt]
+        starts = [(t * T, min(T, nv - t * T)) for t in range(-(-nv // T))]
+        starts += [(nv + t * T, min(T, nt - t * T)) for t in range(-(-nt // T))]
+        ends = np.array([min(j * npf + npf, nv) if j < nv // npf else nv + (j - nv // npf + 1) * npf
+                         for j in range(n_blk)])
+        for a, n in starts:
+            hist = np.nonzero(ends <= a)[0]               # blocks that end before the tile's first row
+            if hist.size == 0:
+                tgt = np.zeros(0, np.int64)
+            else:
+                recent = hist[-CLUSTER_RECENT:]
+                rest = hist[:-CLUSTER_RECENT] if hist.size > CLUSTER_RECENT else hist[:0]
+                pick = rng.choice(rest, size=min(CLUSTER_RANDOM, rest.size), replace=False) if rest.size else rest
+                tgt = np.concatenate([recent, pick])
+            rows = slice(s0 + a, s0 + a + n)
+            noise = np.float32(CLUSTER_QUERY_NOISE) * q[rows]
+            if tgt.size:
+                centre = topic[tgt].sum(axis=0) / np.float32(math.sqrt(tgt.size))   # [hkv, d]
+                q[rows] = noise + np.repeat(centre, gq, axis=0)[None]
+            else:
+                q[rows] = noise
+
+
 def make_probe(cfg: ProbeConfig, layer: int = 0, mask=None) -> Probe:
     """Draw Q/K/V for one layer of ``cfg`` and return them with the mask."""
     if cfg.layers > 1:
@@ -210,6 +263,8 @@ def make_probe(cfg: ProbeConfig, layer: int = 0, mask=None) -> Probe:
         np.divide(x, div, out=x)
     cu = np.zeros(cfg.num_videos + 1, dtype=np.int64)
     cu[1:] = np.cumsum(cfg.seqlens)
+    if cfg.regime == "clustered":
+        _clustered(cfg, q, k, cu, np.random.default_rng([cfg.seed, 7]))
     planted = _planted_frames(cfg)
     gq = cfg.hq // cfg.hkv
     nv_tok = cfg.tokens_per_frame

@@ -302,3 +302,36 @@ def test_coarse_evidence_matches_oracle(cuda_lib, name, block, tau):
                                             head=maps[2].clone(), aqf=maps[3].clone(), accumulate=True)
     check_maps([np32(m) for m in maps2], [2 * w for w in want], probe, label=f"{name} coarse x2")
     ws.free()
+
+
+def test_topp_sparse_regime_long(cuda_lib):
+    """The 65K probe with concentrated attention (long65k_sparse: clustered
+    keys and queries), where tau_p = 0.97 keeps a small share of each row's
+    history, as the retention rule intends. Sampled rows' sets against the
+    float64 oracle; the probe on the tile union with the per-row bits against
+    the oracle restricted to the GPU's own sets, on the same rows."""
+    import torch
+    probe = wl.make_probe(wl.CONFIGS["long65k_sparse"])
+    cfg = probe.cfg
+    block, tau = cfg.tokens_per_frame, 0.97
+    n = int(probe.cu_seqlens[-1])
+    rng = np.random.default_rng(5)
+    rows = np.unique(np.concatenate([[0, 1, 127, 128, n - 1, n - 128, int(probe.n_vis[0])], rng.integers(0, n, 24)]))
+    gpu, keep, uni = _gpu_sets(cuda_lib, probe, block, tau, rows)
+    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, tau, rows=rows)
+    bounds = _logit_bounds(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, block, rows)
+    _check_sets(gpu, probs, bounds, probe.cu_seqlens, probe.n_vis, block, tau, "long65k_sparse")
+    share = [len(ids) / probs[key][0].size for key, ids in gpu.items() if probs[key][0].size >= 64]
+    assert np.median(share) < 0.1, f"not the sparse regime: median kept share {np.median(share):.3f}"
+    row_ptr, col_idx = B.tile_union_to_csr(uni, probe.n_vis, cfg.tile)
+    q, k, v = to_device(probe)
+    o, lse, ws = cuda_lib.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame,
+                                                 cfg.tile, row_ptr, col_idx, keep=keep, keep_block=block)
+    torch.cuda.synchronize()
+    assert cuda_lib.evisel_status(ws) == 0
+    ws.free()
+    kept = _sets_from_keep(keep, rows, probe.cu_seqlens, probe.n_vis, block)
+    o_ref, lse_ref = oracle.probe_rows_topp(probe.q, probe.k, probe.v, probe.cu_seqlens, probe.n_vis, block, kept,
+                                            rows)
+    check_o(o.float().cpu().numpy()[rows], o_ref, "long65k_sparse probe on the top-p masks")
+    check_lse(lse.cpu().numpy()[:, rows], lse_ref, "long65k_sparse probe on the top-p masks")
