@@ -18,6 +18,9 @@
 // adds the spans of each key frame and writes A_ff[a-1, b]. A frame pair
 // (a, b) belongs to exactly one (row tile, kept tile), so every entry has one
 // writer and a fixed summation order (deterministic).
+// Unless it accumulates, the first CTA of each row tile also writes the
+// zeros of its query frames' A_ff rows (entries of key frames the mask does
+// not keep, and b >= a), so no clearing pass runs before it.
 // e_ff_kernel: one CTA per (32 frames, video) forms E_ff from A_ff: the
 // received attention by column sums (32 warps over the rows, coalesced), the
 // given attention by row sums (a warp per frame), partials added in a fixed
@@ -33,10 +36,12 @@ namespace {
 
 constexpr int kUnits = 16;                       // (kept tile, key span) units per CTA
 constexpr unsigned kFull = 0xffffffffu;
+constexpr int kMaxKeptTiles = kCrossFrameMaxKept;   // kept tiles of a row tile that the clearing CTA stages
 
 template <int TILE>
 __global__ void __launch_bounds__(TILE) cross_frame_pairs_kernel(const __grid_constant__ CrossFrameLaunch L) {
   __shared__ float red[TILE / 32][kUnits];
+  __shared__ int kept[kMaxKeptTiles];
   const VisRow R = L.rows[blockIdx.x];
   const int fpt = L.fpt;                           // spans per kv tile (1, 2, 4 or 8; divides kUnits)
   const int u0 = blockIdx.y * kUnits;              // first unit: kept tile u0 / fpt, span u0 % fpt
@@ -48,8 +53,36 @@ __global__ void __launch_bounds__(TILE) cross_frame_pairs_kernel(const __grid_co
   const int row = threadIdx.x, lane = row & 31, warp = row >> 5;
   const bool valid = row < R.q_len;
   const int a = (R.row_tile * TILE + row) / npf;   // the row's frame (video-local)
+  // Overwrite mode: the first CTA of each row tile writes the zeros of its
+  // query frames' rows of A_ff, the entries no CTA writes (key frames of tiles
+  // the mask does not keep, and b >= a), so the call needs no clearing pass.
+  // The entries it writes and the ones the pairs below write are disjoint.
+  if (!L.accumulate && blockIdx.y == 0 && R.kv_count <= kMaxKeptTiles) {
+    for (int i = threadIdx.x; i < R.kv_count; i += TILE)
+      kept[i] = (L.kv[R.kv_begin + i].start - vi.vis_start) / TILE;
+    __syncthreads();
+    const int a0 = max(1, (R.row_tile * TILE) / npf);
+    const int a1 = min(T, (R.row_tile * TILE + R.q_len) / npf);   // frames [a0, a1) of this row tile
+    for (int a_ = a0; a_ < a1; ++a_) {
+      float* arow = L.aff + L.aff_off[R.video] + static_cast<int64_t>(a_ - 1) * (T - 1);
+      for (int b = threadIdx.x; b < T - 1; b += TILE) {
+        bool written = false;
+        if (b < a_) {
+          const int tb = b * npf / TILE;           // the key frame's tile: kept? (the list is sorted)
+          int lo = 0, hi = R.kv_count;
+          while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (kept[mid] < tb) lo = mid + 1; else hi = mid;
+          }
+          written = lo < R.kv_count && kept[lo] == tb;
+        }
+        if (!written) arow[b] = 0.f;
+      }
+    }
+  }
   // Units u0 .. u0 + 15 are consecutive spans of consecutive kept tiles: for a
-  // head they are one contiguous run of 16 x TILE floats.
+  // head they are one contiguous run of 16 x TILE floats. Two heads at a time,
+  // so that 32 loads of a thread are in flight.
   float v[kUnits];
 #pragma unroll
   for (int u = 0; u < kUnits; ++u) v[u] = 0.f;
@@ -79,7 +112,7 @@ __global__ void __launch_bounds__(TILE) cross_frame_pairs_kernel(const __grid_co
 #pragma unroll
       for (int u = 0; u < kUnits; ++u) red[warp][u] = v[u];
     }
-    __syncthreads();
+    __syncthreads();   // uniform: every thread of the CTA gets here
     if (row % npf == 0) {
 #pragma unroll
       for (int u = 0; u < kUnits; ++u) {

@@ -335,9 +335,21 @@ void build_plan(const evisel_probe_args* a, Plan& P) {
     }
   }
   // Longest first; stable so that the heads of one row tile stay adjacent and
-  // share their K/V tiles through L2.
-  std::stable_sort(items.begin(), items.end(),
-                   [](const WorkItem& x, const WorkItem& y) { return x.kv_count > y.kv_count; });
+  // share their K/V tiles through L2. A probe on top-p masks (keep bits) runs
+  // over tile unions that cover most of each row's causal history: there the
+  // items go KV group by group (longest first within a group), so that the
+  // CTAs in flight read one group's K/V (33.5 MB at 65K tokens), which L2
+  // holds, instead of all groups' (A/B on 65K tokens: same time, static mask
+  // or union; the static masks keep the plain order).
+  if (a->keep) {
+    std::stable_sort(items.begin(), items.end(), [gq](const WorkItem& x, const WorkItem& y) {
+      const int gx = x.head / gq, gy = y.head / gq;
+      return gx != gy ? gx < gy : x.kv_count > y.kv_count;
+    });
+  } else {
+    std::stable_sort(items.begin(), items.end(),
+                     [](const WorkItem& x, const WorkItem& y) { return x.kv_count > y.kv_count; });
+  }
   P.items = std::move(items);
 
   // Evidence column chunks.
@@ -411,7 +423,7 @@ namespace {
 
 std::vector<int32_t> plan_key(const evisel_probe_args* a) {
   std::vector<int32_t> k = {a->num_videos, a->tokens_per_frame, a->hq, a->hkv, a->head_dim, a->tile, a->cross_frame,
-                            a->text_evidence};
+                            a->text_evidence, a->keep != nullptr};   // the item order differs with keep bits
   for (int b = 0; b <= a->num_videos && a->num_videos > 0; ++b) k.push_back(a->cu_seqlens_h[b]);
   for (int b = 0; b < a->num_videos; ++b) k.push_back(a->n_vis_h[b]);
   int64_t rows = 0;
@@ -760,7 +772,9 @@ int evisel_cross_frame_evidence(const evisel_probe_args* args, evisel_ws* ws, fl
     cudaError_t e = cudaStreamWaitEvent(stream, ws->stage_done, 0);
     if (e != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
   }
-  if (!accumulate && P.aff_floats > 0) {
+  // Without accumulate the pairs kernel writes every entry of A_ff (zeros
+  // included) when no row tile keeps more tiles than it stages; else clear first.
+  if (!accumulate && P.aff_floats > 0 && P.max_kv > kCrossFrameMaxKept) {
     cudaError_t e = cudaMemsetAsync(aff, 0, static_cast<size_t>(P.aff_floats) * sizeof(float), stream);
     if (e != cudaSuccess) return cuda_fail(e, "A_ff clear");
   }

@@ -155,6 +155,10 @@ struct VisRow {
 };
 static_assert(sizeof(VisRow) == 32, "VisRow is 32 bytes");
 
+// Kept tiles per row tile up to which the cross-frame pairs kernel also
+// writes the zeros of A_ff (beyond it the entry point clears A_ff first).
+constexpr int kCrossFrameMaxKept = 1024;
+
 struct CrossFrameLaunch {
   const VisRow* rows;
   const KvTile* kv;

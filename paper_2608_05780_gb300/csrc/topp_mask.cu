@@ -16,13 +16,13 @@
 //   warp / 4). The heads of the group go in pairs: S = Q_h k_bar^T for both
 //   heads of a pair, in chunks of 128 blocks (tcgen05, both products from one
 //   k_bar chunk, TMEM 2 buffers x 2 heads), in six passes over the chunks:
-//     0     the row's max and min logit over H_i and the softmax sum Z (online);
+//     0     the row's max and min logit over H_i;
 //     1..4  a radix select on the block's key q = floor((max - x) 2^14 / (max -
 //           min)) (0 = the largest logit), digit by digit (3, 3, 4 and 4 bits,
 //           top first): the mass per digit value of the blocks whose higher
-//           digits equal the boundary's, in 8 or 16 register bins; the boundary
-//           digit is the one where the cumulative mass from the top reaches
-//           tau_p Z;
+//           digits equal the boundary's, in 8 or 16 register bins (the first
+//           digit's bins together give the softmax sum Z); the boundary digit
+//           is the one where the cumulative mass from the top reaches tau_p Z;
 //     5     keep every block whose key is below the boundary key; at the
 //           boundary key, blocks in id order while the mass before them is
 //           below tau_p Z.
@@ -301,6 +301,8 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
               ptx::tmem_wait_ld();
               const int jn = nh - (ch * kCols + c0);         // columns e < jn are in H_i
               if (pass == 0) {
+                // The row's max and min over H_i (the softmax sum comes from the
+                // first digit's bins, which every block of H_i falls in).
                 float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
                 float mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
 #pragma unroll
@@ -311,17 +313,8 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
                     mn[e & 3] = fminf(mn[e & 3], x);
                   }
                 }
-                const float cmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+                m = fmaxf(m, fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])));
                 gmin = fminf(gmin, fminf(fminf(mn[0], mn[1]), fminf(mn[2], mn[3])));
-                if (cmax > m) {
-                  z = (m == -INFINITY) ? 0.f : z * ptx::ex2(m - cmax);
-                  m = cmax;
-                }
-                float zs[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-                for (int e = 0; e < 32; ++e)
-                  if (e < jn) zs[e & 3] += ptx::ex2(__fsub_rn(__fmul_rn(__uint_as_float(r[e]), sc), m));
-                z += (zs[0] + zs[1]) + (zs[2] + zs[3]);
               } else if (lv == 0) {
                 // The first digit (every column is in the window): no branches,
                 // so that the columns' arithmetic overlaps.
@@ -402,9 +395,14 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
         // the total below it (tau_p near 1), the last non-empty one, whose
         // blocks are then all kept.
         if (pass == 0) {
-          target = L.tau * z;
           inv_r = static_cast<float>(kQMax + 1) / fmaxf(m - gmin, 1e-30f);
         } else if (lv < kLevels) {
+          if (lv == 0) {
+            // Z: the first digit's bins hold the weight of every block of H_i.
+#pragma unroll
+            for (int kb = 0; kb < 8; ++kb) z += acc[kb];
+            target = L.tau * z;
+          }
           float run = above, before_last = above;
           int found = -1, last = 0;
 #pragma unroll
