@@ -199,7 +199,9 @@ const char* evisel_build_id(void);
  *     without ordering) race on the array: order them on one stream.
  *   - device_status: NULL -> the call is asynchronous on `stream`; otherwise it
  *     waits for `stream` and stores the device status word there (EVISEL_OK or
- *     EVISEL_ETIMEOUT).
+ *     EVISEL_ETIMEOUT). With NULL a device-side timeout is not reported: the
+ *     status word lives in the shared array, no other call reads it, and the
+ *     next call clears it. Callers that need to know pass a pointer.
  * Errors: as evisel_probe_attention() and evisel_evidence_reduce(). */
 #define EVISEL_NOALLOC_SCRATCH_BYTES (64LL << 20)
 int evisel_probe_evidence_noalloc(const evisel_probe_args* args, float* tok, float* frame, float* head,
