@@ -200,25 +200,37 @@ __device__ __forceinline__ void mma_issuer(const ProbeLaunch& L, const WorkItem&
     same_leader = same_leader && static_cast<int>(leader) == first_leader;
     return me && same_leader;
   };
+  // Descriptors of every operand buffer, built once; a k-step adds its byte
+  // offset / 16 to the address field (the lowest bits; smem offsets < 256 KB
+  // never carry out of it).
+  const uint64_t dq0 = ptx::sdesc_sw128(sbase + C::OFF_Q, 16, 1024);
+  const uint64_t dq1 = ptx::sdesc_sw128(sbase + C::OFF_Q + C::Q_BYTES, 16, 1024);
+  const uint64_t dk0 = ptx::sdesc_sw128(sbase + C::OFF_K, 16, 1024);
+  const uint64_t dk1 = ptx::sdesc_sw128(sbase + C::OFF_K + C::KV_BYTES, 16, 1024);
+  const uint64_t dv0 = ptx::sdesc_sw128(sbase + C::OFF_V, C::KV_BLOCK, 1024);
+  const uint64_t dv1 = ptx::sdesc_sw128(sbase + C::OFF_V + C::KV_BYTES, C::KV_BLOCK, 1024);
+  static_assert(NS == 2, "two ring stages");
   // S[buf] = Q_slot K_j^T (buf: whose S columns receive it)
   auto mma_s = [&](int slot, int j, int buf) {
-    const uint32_t kbase = sbase + C::OFF_K + (j % NS) * C::KV_BYTES;
-    const uint32_t qbase = sbase + C::OFF_Q + slot * C::Q_BYTES;
+    const uint64_t qd = slot ? dq1 : dq0;
+    const uint64_t kd = (j & 1) ? dk1 : dk0;
+    const uint32_t d_tmem = tmem + buf * C::SLOT_COLS + C::COL_S;
 #pragma unroll
     for (int kk = 0; kk < D / 16; ++kk) {
-      const uint64_t a = ptx::sdesc_sw128(qbase + (kk / 4) * C::Q_BLOCK + (kk % 4) * 32, 16, 1024);
-      const uint64_t bd = ptx::sdesc_sw128(kbase + (kk / 4) * C::KV_BLOCK + (kk % 4) * 32, 16, 1024);
-      ptx::mma_ss(tmem + buf * C::SLOT_COLS + C::COL_S, a, bd, kIdescS, kk > 0 ? 1u : 0u);
+      const uint64_t a = qd + static_cast<uint64_t>(((kk / 4) * C::Q_BLOCK + (kk % 4) * 32) >> 4);
+      const uint64_t bd = kd + static_cast<uint64_t>(((kk / 4) * C::KV_BLOCK + (kk % 4) * 32) >> 4);
+      ptx::mma_ss(d_tmem, a, bd, kIdescS, kk > 0 ? 1u : 0u);
     }
   };
   // O_slot += P V_j, P from the first TILE/2 columns of S[buf].
   auto mma_pv = [&](int slot, int j, int buf) {
-    const uint32_t vbase = sbase + C::OFF_V + (j % NS) * C::KV_BYTES;
+    const uint64_t vd = (j & 1) ? dv1 : dv0;
+    const uint32_t d_tmem = tmem + slot * C::SLOT_COLS + C::COL_O;
+    const uint32_t p_tmem = tmem + buf * C::SLOT_COLS + C::COL_S;
 #pragma unroll
     for (int kk = 0; kk < TILE / 16; ++kk) {
-      const uint64_t bd = ptx::sdesc_sw128(vbase + kk * 16 * 128, C::KV_BLOCK, 1024);
-      ptx::mma_ts(tmem + slot * C::SLOT_COLS + C::COL_O, tmem + buf * C::SLOT_COLS + C::COL_S + kk * 8, bd, kIdescO,
-                  (j > 0 || kk > 0) ? 1u : 0u);
+      const uint64_t bd = vd + static_cast<uint64_t>((kk * 16 * 128) >> 4);
+      ptx::mma_ts(d_tmem, p_tmem + kk * 8, bd, kIdescO, (j > 0 || kk > 0) ? 1u : 0u);
     }
   };
 

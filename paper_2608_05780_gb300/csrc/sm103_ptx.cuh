@@ -63,13 +63,13 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const v
 
 // ---------------------------------------------------------------- warp
 // Elects one lane of a converged warp (elect.sync); every lane learns which
-// one through a ballot.
+// one (elect.sync returns the elected lane id to all of them).
 __device__ __forceinline__ bool elect_one(uint32_t& leader) {
-  uint32_t pred;
+  uint32_t pred, lane_id;
   asm volatile(
-      "{\n\t.reg .pred P;\n\telect.sync _|P, 0xffffffff;\n\tselp.b32 %0, 1, 0, P;\n\t}"
-      : "=r"(pred));
-  leader = static_cast<uint32_t>(__ffs(__ballot_sync(0xffffffffu, pred != 0)) - 1);
+      "{\n\t.reg .pred P;\n\telect.sync %1|P, 0xffffffff;\n\tselp.b32 %0, 1, 0, P;\n\t}"
+      : "=r"(pred), "=r"(lane_id));
+  leader = lane_id;
   return pred != 0;
 }
 
