@@ -23,8 +23,8 @@
 // not keep, and b >= a), so no clearing pass runs before it.
 // e_ff_kernel: one CTA per (32 frames, video) forms E_ff from A_ff: the
 // received attention by column sums (32 warps over the rows, coalesced), the
-// given attention by row sums (a warp per frame), partials added in a fixed
-// order.
+// given attention by row sums (a warp per frame); each lane keeps 16 loads in
+// flight over four partial sums, and every partial is added in a fixed order.
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -155,11 +155,24 @@ __global__ void __launch_bounds__(kEffWarps * 32) e_ff_kernel(const __grid_const
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int t = t0 + lane;
   // Received: column t over the rows of frames a > t (row index a - 1 >= t).
+  // Four partial sums, 16 loads in flight per lane, added in a fixed order.
   float recv = 0.f;
   if (t <= T - 2) {
-#pragma unroll 4
-    for (int ra = t0 + warp; ra <= T - 2; ra += kEffWarps)
-      if (ra >= t) recv += A[static_cast<int64_t>(ra) * (T - 1) + t];
+    float r4[4] = {0.f, 0.f, 0.f, 0.f};
+    int ra = t0 + warp;
+    for (; ra + 15 * kEffWarps <= T - 2; ra += 16 * kEffWarps) {
+      float x[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int rr = ra + i * kEffWarps;
+        x[i] = rr >= t ? A[static_cast<int64_t>(rr) * (T - 1) + t] : 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < 16; ++i) r4[i & 3] += x[i];
+    }
+    for (; ra <= T - 2; ra += kEffWarps)
+      if (ra >= t) r4[0] += A[static_cast<int64_t>(ra) * (T - 1) + t];
+    recv = (r4[0] + r4[1]) + (r4[2] + r4[3]);
   }
   part[warp][lane] = recv;
   // Given: row t - 1 over the frames b < t, one warp per frame.
@@ -167,8 +180,18 @@ __global__ void __launch_bounds__(kEffWarps * 32) e_ff_kernel(const __grid_const
     const int tg = t0 + warp;
     float g = 0.f;
     if (tg >= 1 && tg < T) {
-#pragma unroll 4
-      for (int b = lane; b < tg; b += 32) g += A[static_cast<int64_t>(tg - 1) * (T - 1) + b];
+      const float* row = A + static_cast<int64_t>(tg - 1) * (T - 1);
+      float g4[4] = {0.f, 0.f, 0.f, 0.f};
+      int b = lane;
+      for (; b + 15 * 32 < tg; b += 16 * 32) {
+        float x[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) x[i] = row[b + i * 32];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) g4[i & 3] += x[i];
+      }
+      for (; b < tg; b += 32) g4[0] += row[b];
+      g = (g4[0] + g4[1]) + (g4[2] + g4[3]);
     }
     for (int off = 16; off > 0; off >>= 1) g += __shfl_xor_sync(kFull, g, off);
     if (lane == 0) give[warp] = g;
