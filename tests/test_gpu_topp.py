@@ -176,6 +176,32 @@ def test_topp_edge_cases(cuda_lib, name, block, tau):
     _check_sets(gpu, probs, bounds, probe.cu_seqlens, probe.n_vis, block, min(tau, 1.0 - 1e-6), name)
 
 
+@pytest.mark.parametrize("tau", [0.97, 0.5, 1.0])
+def test_topp_window_overflow(cuda_lib, tau):
+    """Rows whose boundary window holds more blocks than a row's list: heads 0
+    and 1 (one pair of KV group 0) have q = 0, so every block of H_i ties and
+    rows with more than 32 blocks flag the pair for the radix path; heads 2-5
+    keep their random q (the fast path, in the same CTAs). With all logits
+    equal, S_i is the first ceil(tau |H_i|) blocks by id."""
+    from test_gpu_parity import _custom
+    probe = _custom(frames=(80,), n_text=(40,), npf=16, hq=6, hkv=2, d=64, tile=64, window=2, seed=11)
+    probe.q[:, :2, :] = 0.0
+    rows = _all_rows(probe)
+    gpu, _, _ = _gpu_sets(cuda_lib, probe, 16, tau, rows)
+    _, probs = oracle.retained_blocks(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, 16, tau, rows=rows)
+    bounds = _logit_bounds(probe.q, probe.k, probe.cu_seqlens, probe.n_vis, 16, rows)
+    _check_sets(gpu, probs, bounds, probe.cu_seqlens, probe.n_vis, 16, min(tau, 1.0 - 1e-6), "overflow")
+    n_long = 0
+    for row in rows:
+        hist, _ = probs[(0, int(row))]
+        n_long += hist.size > 32
+        for h in (0, 1):
+            own = int(row) // 16 if row < 1280 else 80 + (int(row) - 1280) // 16
+            want = list(range(math.ceil(tau * hist.size - 1e-9))) if hist.size else []
+            assert sorted(set(gpu[(h, int(row))]) - {own}) == want, (tau, h, int(row))
+    assert n_long > 500       # most rows take the radix path
+
+
 def test_topp_union_drives_the_probe(cuda_lib):
     """The tile union equals the union of the GPU's own sets; as a mask it runs the probe."""
     import torch
