@@ -799,6 +799,7 @@ int evisel_cross_frame_evidence(const evisel_probe_args* args, evisel_ws* ws, fl
   L.n_tok = P.n_tok;
   L.hq = args->hq;
   L.accumulate = accumulate != 0;
+  L.status = ws->status;
   cudaError_t e = launch_cross_frame(L, stream);
   if (e != cudaSuccess) return cuda_fail(e, "cross_frame launch");
   ws->last_stream = stream;

@@ -174,6 +174,7 @@ struct CrossFrameLaunch {
   int spans_per_frame;              // N_v / span
   int n_tok, hq;
   int accumulate;
+  int* status;                      // device status word (a timed-out wait records EVISEL_ETIMEOUT)
 };
 
 // Text-row evidence by recompute (no logit spill): one CTA per (128 visual

@@ -35,8 +35,9 @@
 //   digit value in register bins; then every block whose key is below the
 //   boundary key is kept and, at the boundary key, blocks in id order while the
 //   mass before them is below tau_p Z.
-// topp_union_kernel: one thread per (row, head) ORs its bits, mapped to key
-//   tiles, into its attention row tile's union.
+// topp_union_kernel: per (visual row tile, 1,024 blocks) the OR of the rows'
+//   bits over the heads, folded into key tiles, as its attention row tiles'
+//   union words.
 // Every wait is bounded; a timeout records EVISEL_ETIMEOUT.
 #include <cstdint>
 #include <cuda_bf16.h>
@@ -226,6 +227,7 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
     uint32_t leader = 0;
     int nq = 0, nk = 0;                          // Q (per pair job) and k_bar loads issued
     auto job = [&](int pair, int passes) -> bool {
+      if (n_ch == 0) return true;                // no block ends before the tile's rows: nothing to load
       if (nq >= 1 && !warp_wait(bar(C::B_QE), (nq - 1) & 1, abort_flag)) return false;
       const int nheads = min(kHeadSlots, gq - pair * kHeadSlots);
       if (ptx::elect_one(leader)) {
@@ -275,6 +277,7 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
     int first_leader = -1, nj = 0, t = 0;
     bool same = true, issued = false;
     auto job = [&](int pair, int passes) -> bool {
+      if (n_ch == 0) return true;                // as the producer: no Q, no steps
       const int nheads = min(kHeadSlots, gq - pair * kHeadSlots);
       for (int s = 0; s < passes * n_ch; ++s, ++t) {
         const int b = t % 2;
@@ -730,45 +733,98 @@ __global__ void __launch_bounds__(kThreads, 1) topp_select_kernel(const __grid_c
   }
 }
 
+// Keeps bit 0 of every BPT-bit group of x (the group's OR after or_fold),
+// packed into the low 32 / BPT bits.
+template <int BPT>
+__device__ __forceinline__ uint32_t or_fold(uint32_t x) {
+#pragma unroll
+  for (int k = 1; k < BPT; k <<= 1) x |= x >> k;
+  return x;
+}
+template <int BPT>
+__device__ __forceinline__ uint32_t compress(uint32_t x) {
+  if constexpr (BPT == 1) {
+    return x;
+  } else if constexpr (BPT == 2) {
+    x &= 0x55555555u;
+    x = (x | (x >> 1)) & 0x33333333u;
+    x = (x | (x >> 2)) & 0x0f0f0f0fu;
+    x = (x | (x >> 4)) & 0x00ff00ffu;
+    return (x | (x >> 8)) & 0x0000ffffu;
+  } else if constexpr (BPT == 4) {
+    x &= 0x11111111u;
+    x = (x | (x >> 3)) & 0x03030303u;
+    x = (x | (x >> 6)) & 0x000f000fu;
+    return (x | (x >> 12)) & 0x000000ffu;
+  } else {
+    static_assert(BPT == 8, "blocks per key tile: 1, 2, 4 or 8");
+    x &= 0x01010101u;
+    x = (x | (x >> 7)) & 0x00030003u;
+    return (x | (x >> 14)) & 0x0000000fu;
+  }
+}
+
+constexpr int kUnionWords = 32;                  // keep words (1,024 blocks) per union CTA
+
+// blockIdx.x: builder row tile (visual rows), blockIdx.y: a chunk of 32 keep
+// words, i.e. 32 / BPT words of the union. A thread ORs its row's words over
+// the heads (32 independent loads per head), masks them to the visual blocks,
+// folds blocks into key tiles, the warps OR their rows (shuffles, then shared
+// memory), and one thread stores each union word of each attention row tile
+// the CTA covers (one writer per word: no atomics).
+template <int BPT>
 __global__ void __launch_bounds__(128) topp_union_kernel(const __grid_constant__ ToppLaunch L) {
-  // blockIdx.x: builder row tile, blockIdx.y: head; one thread per row. Word
-  // by word of the union (32 key tiles = 32 * tile / block blocks), a thread
-  // folds its blocks into tile bits, the warp ORs them, one lane stores.
+  constexpr int kTileWords = kUnionWords / BPT;
+  __shared__ uint32_t part[4][kTileWords];
   const ToppRowTile rt = L.tiles[blockIdx.x];
   if (rt.text) return;                           // the attention takes tile masks for visual rows only
   const ToppVideo vid = L.vids[rt.video];
-  const int h = blockIdx.y, row = threadIdx.x;
-  const int pos = rt.local0 + min(row, rt.q_len - 1);
-  const bool row_ok = row < rt.q_len;
-  const int bpt = L.tile / L.block;              // blocks per key tile: 1, 2, 4 or 8
   const int nvb = vid.n_vis / L.block;           // visual blocks (visual rows keep no text block)
-  const int n_vt = (vid.n_vis + L.tile - 1) / L.tile;
-  const uint32_t* keep = L.keep + static_cast<int64_t>(h) * L.n_words * L.n_tok + vid.start + pos;
-  // Rows of one warp may belong to two attention row tiles (tile = 64): reduce per tile.
-  const int my_tile = pos / L.tile;
-  for (int tw = 0; tw * 32 < n_vt; ++tw) {
+  const int w0 = blockIdx.y * kUnionWords;
+  if (w0 * 32 >= nvb) return;                    // uniform: no visual block in this chunk
+  const int row = threadIdx.x, lane = row & 31, warp = row >> 5;
+  const bool row_ok = row < rt.q_len;
+  uint32_t acc[kUnionWords];
+#pragma unroll
+  for (int i = 0; i < kUnionWords; ++i) acc[i] = 0u;
+  if (row_ok) {
+    const uint32_t* kp = L.keep + static_cast<int64_t>(w0) * L.n_tok + rt.q_start + row;
+    for (int h = 0; h < L.hq; ++h) {
+      const uint32_t* kh = kp + static_cast<int64_t>(h) * L.n_words * L.n_tok;
+#pragma unroll
+      for (int i = 0; i < kUnionWords; ++i)
+        if (w0 + i < L.n_words) acc[i] |= kh[static_cast<int64_t>(i) * L.n_tok];
+    }
+  }
+  uint32_t tw[kTileWords];
+#pragma unroll
+  for (int j = 0; j < kTileWords; ++j) {
     uint32_t bits = 0u;
-    if (row_ok) {
-      for (int q = 0; q < bpt; ++q) {            // keep words tw * bpt + q: blocks of tiles 32 tw + (32 q .. 32 q + 31) / bpt
-        const int w = tw * bpt + q;
-        if (w >= L.n_words || w * 32 >= nvb) break;
-        uint32_t x = keep[static_cast<int64_t>(w) * L.n_tok];
-        if (w * 32 + 32 > nvb) x &= (1u << (nvb - w * 32)) - 1u;   // visual blocks only
-        for (int k = 1; k < bpt; k <<= 1) x |= x >> k;             // a tile's OR in its lowest block bit
-        for (int i = 0; i < 32 / bpt; ++i)
-          if ((x >> (i * bpt)) & 1u) bits |= 1u << (q * (32 / bpt) + i);
-      }
+#pragma unroll
+    for (int q = 0; q < BPT; ++q) {
+      const int i = j * BPT + q, b0 = (w0 + i) * 32;   // blocks b0 .. b0 + 31
+      uint32_t x = acc[i];
+      if (b0 + 32 > nvb) x &= b0 < nvb ? (1u << (nvb - b0)) - 1u : 0u;
+      bits |= compress<BPT>(or_fold<BPT>(x)) << (q * (32 / BPT));
     }
-    const int lane = threadIdx.x & 31;
-    const int first_tile = __shfl_sync(0xffffffffu, my_tile, 0);
-    const bool one_tile = __all_sync(0xffffffffu, my_tile == first_tile);
-    if (one_tile) {
-      const uint32_t wbits = __reduce_or_sync(0xffffffffu, bits);
-      if (lane == 0 && wbits)
-        atomicOr(L.tile_union + static_cast<int64_t>(vid.row_tile0 + my_tile) * L.n_tile_words + tw, wbits);
-    } else if (bits) {
-      atomicOr(L.tile_union + static_cast<int64_t>(vid.row_tile0 + my_tile) * L.n_tile_words + tw, bits);
-    }
+    tw[j] = __reduce_or_sync(0xffffffffu, bits);
+  }
+  // Attention row tiles: TILE = 128 is the CTA's rows; TILE = 64 gives warps
+  // 0-1 and 2-3 a tile each (the builder's tiles start at multiples of 128).
+  if (lane == 0) {
+#pragma unroll
+    for (int j = 0; j < kTileWords; ++j) part[warp][j] = tw[j];
+  }
+  __syncthreads();
+  const int wpt = L.tile / 32;                   // warps per attention row tile
+  const int n_at = (rt.q_len + L.tile - 1) / L.tile;
+  const int t = threadIdx.x / kTileWords, j = threadIdx.x % kTileWords;
+  if (t < n_at) {
+    uint32_t bits = 0u;
+    for (int ww = t * wpt; ww < (t + 1) * wpt; ++ww) bits |= part[ww][j];
+    const int tile_word = w0 / BPT + j;
+    if (tile_word < L.n_tile_words)
+      L.tile_union[static_cast<int64_t>(vid.row_tile0 + rt.local0 / L.tile + t) * L.n_tile_words + tile_word] = bits;
   }
 }
 
@@ -799,8 +855,13 @@ cudaError_t launch_topp(const ToppLaunch& L, cudaStream_t stream) {
                                     : cudaErrorInvalidValue;
   if (e != cudaSuccess) return e;
   if (L.tile_union) {
-    dim3 grid(L.n_tiles, L.hq);
-    topp_union_kernel<<<grid, 128, 0, stream>>>(L);
+    dim3 grid(L.n_tiles, (L.n_words + kUnionWords - 1) / kUnionWords);
+    const int bpt = L.tile / L.block;
+    if (bpt == 1) topp_union_kernel<1><<<grid, 128, 0, stream>>>(L);
+    else if (bpt == 2) topp_union_kernel<2><<<grid, 128, 0, stream>>>(L);
+    else if (bpt == 4) topp_union_kernel<4><<<grid, 128, 0, stream>>>(L);
+    else if (bpt == 8) topp_union_kernel<8><<<grid, 128, 0, stream>>>(L);
+    else return cudaErrorInvalidValue;
     return cudaGetLastError();
   }
   return cudaSuccess;

@@ -202,6 +202,45 @@ def test_topp_window_overflow(cuda_lib, tau):
     assert n_long > 500       # most rows take the radix path
 
 
+UNION_CASES = {
+    # (probe, block): blocks per key tile 8, 4, 2 and 1; tiles of 64 and 128; ragged tiles, packed videos
+    "single_b16": ("single", None, 16),
+    "t128_b32": (None, dict(frames=(30,), n_text=(25,), npf=32, hq=4, hkv=2, d=64, tile=128, window=2), 32),
+    "t64_b16": (None, dict(frames=(23,), n_text=(30,), npf=16, hq=4, hkv=2, d=64, tile=64, window=2), 16),
+    "t64_b64": (None, dict(frames=(21,), n_text=(17,), npf=64, hq=4, hkv=2, d=64, tile=64, window=2), 64),
+    "t128_b64": (None, dict(frames=(3, 9, 14), n_text=(20, 0, 45), npf=64, hq=6, hkv=2, d=128, tile=128,
+                            window=2), 64),
+    "t128_b128": (None, dict(frames=(13, 6), n_text=(40, 9), npf=128, hq=4, hkv=1, d=128, tile=128, window=2), 128),
+    # 1,280 visual blocks: the union's second chunk of 1,024 blocks
+    "t128_b16_two_chunks": (None, dict(frames=(80,), n_text=(20,), npf=16, hq=4, hkv=2, d=64, tile=128, window=2), 16),
+}
+
+
+@pytest.mark.parametrize("case", sorted(UNION_CASES))
+def test_topp_union_matches_the_sets(cuda_lib, case):
+    """The tile union, bit for bit, against the union of the GPU's own sets of
+    every visual row and head, folded into key tiles."""
+    from test_gpu_parity import _custom
+    name, custom, block = UNION_CASES[case]
+    probe = wl.make_probe(wl.CONFIGS[name]) if name else _custom(**custom)
+    cfg = probe.cfg
+    rows = _all_rows(probe)
+    gpu, _, uni = _gpu_sets(cuda_lib, probe, block, 0.6, rows)
+    row_ptr, col_idx = B.tile_union_to_csr(uni, probe.n_vis, cfg.tile)
+    bpt = cfg.tile // block
+    r0 = 0
+    for b in range(len(probe.n_vis)):
+        s0, nv = int(probe.cu_seqlens[b]), int(probe.n_vis[b])
+        n_vt = -(-nv // cfg.tile)
+        want = [set() for _ in range(n_vt)]
+        for (h, row), ids in gpu.items():
+            if s0 <= row < s0 + nv:
+                want[(row - s0) // cfg.tile] |= {j // bpt for j in ids if j < nv // block}
+        for r in range(n_vt):
+            assert sorted(want[r]) == list(col_idx[row_ptr[r0 + r]:row_ptr[r0 + r + 1]]), (case, b, r)
+        r0 += n_vt
+
+
 def test_topp_union_drives_the_probe(cuda_lib):
     """The tile union equals the union of the GPU's own sets; as a mask it runs the probe."""
     import torch
