@@ -157,21 +157,27 @@ __global__ void __launch_bounds__(TILE + 32) cross_frame_pairs_kernel(const __gr
           const float m = mq[i] * 1.4426950408889634f;
           mq[i] = h + 4 < L.hq ? __ldg(lse + static_cast<int64_t>(h + 4) * L.n_tok) : 0.f;
           const int st = h % kStages;
-          ok = ok && __all_sync(kFull, ptx::mbar_wait(full(st), (h / kStages) & 1, &abort_flag, kWaitTimeoutNs));
-          if (ok && valid) {
+          // A warp that gives up releases no more stages: the producer stops
+          // on the abort flag and waits only for the copies it has issued.
+          const bool got =
+              ok && __all_sync(kFull, ptx::mbar_wait(full(st), (h / kStages) & 1, &abort_flag, kWaitTimeoutNs));
+          if (ok && !got) {
+            ok = false;
+            if (lane == 0) {
+              abort_flag = 1;
+              atomicExch(L.status, kStatusTimeout);
+            }
+          }
+          if (got && valid) {
             const float* sr = ring + st * kUnits * TILE + row;
 #pragma unroll
             for (int u = 0; u < kUnits; ++u)
               if (u < n_u) v[u] += ptx::ex2(sr[u * TILE] - m);
           }
           __syncwarp();
-          if (lane == 0) ptx::mbar_arrive(empty(st));
+          if (got && lane == 0) ptx::mbar_arrive(empty(st));
         }
       }
-    }
-    if (!ok && lane == 0) {
-      abort_flag = 1;
-      atomicExch(L.status, kStatusTimeout);
     }
   }
   // Spans -> key frames (spf consecutive units), then sums over the N_v rows

@@ -422,8 +422,42 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
   bool ok = true;
   const uint64_t scale2 = ptx::f2(L.scale_log2, L.scale_log2);
 
+  // With per-row masks (EMB) the kv tiles are read two tiles ahead and the
+  // row's mask word one tile ahead, so that no global load waits between an
+  // S-ready wait and the softmax that follows it. Without them the tile is
+  // read before its S-ready wait, which covers the load.
+  auto load_kv = [&](int jj) { return jj < it.kv_count ? L.kv[it.kv_begin + jj] : KvTile{0, 0, 0, 0}; };
+  [[maybe_unused]] auto mask_word = [&](const KvTile& t) -> uint32_t {
+    uint32_t w = 0xffffffffu;   // bit q: the tile's q-th block is attended
+    if constexpr (EMB > 0) {
+      if (em_row) {
+        const int blk0 = t.visual ? (t.start - em_vis_start) / EMB
+                                  : em_n_vis / EMB + (t.start - em_vis_start - em_n_vis) / EMB;
+        w = em_row[static_cast<int64_t>(blk0 >> 5) * L.n_tok] >> (blk0 & 31);
+      }
+    }
+    return w;
+  };
+  [[maybe_unused]] KvTile kv_next{0, 0, 0, 0}, kv_after{0, 0, 0, 0};
+  [[maybe_unused]] uint32_t em_next = 0xffffffffu;
+  if constexpr (EMB > 0) {
+    kv_next = load_kv(0);
+    kv_after = load_kv(1);
+    if (it.kv_count > 0) em_next = mask_word(kv_next);
+  }
+
   for (int j = 0; j < it.kv_count; ++j) {
-    const KvTile kv = L.kv[it.kv_begin + j];
+    KvTile kv;
+    [[maybe_unused]] uint32_t em_bits = 0xffffffffu;
+    if constexpr (EMB > 0) {
+      kv = kv_next;
+      em_bits = em_next;
+      kv_next = kv_after;
+      if (j + 1 < it.kv_count) em_next = mask_word(kv_next);   // kv_next was read a tile ago
+      kv_after = load_kv(j + 2);
+    } else {
+      kv = L.kv[it.kv_begin + j];
+    }
     const int b = two ? slot : (j & 1);
     const uint32_t par = two ? (j & 1) : ((j >> 1) & 1);
     const uint32_t tS = tmem_base + lane_base + b * C::SLOT_COLS + C::COL_S;
@@ -438,14 +472,6 @@ __device__ __forceinline__ void softmax_epilogue(const ProbeLaunch& L, const Wor
     }
     const bool spill = spill_rows && kv.visual;
     float* spill_dst = spill ? spill_row + static_cast<int64_t>(kv.start - vis_start) * 32 : nullptr;
-    [[maybe_unused]] uint32_t em_bits = 0xffffffffu;   // bit q: the tile's q-th block is attended
-    if constexpr (EMB > 0) {
-      if (em_row) {
-        const int blk0 = kv.visual ? (kv.start - em_vis_start) / EMB
-                                   : em_n_vis / EMB + (kv.start - em_vis_start - em_n_vis) / EMB;
-        em_bits = em_row[static_cast<int64_t>(blk0 >> 5) * L.n_tok] >> (blk0 & 31);
-      }
-    }
     auto apply_em = [&](float* sv, int h) {
       if constexpr (EMB > 0) {
         if ((em_bits & ((1u << (TILE / EMB)) - 1u)) != (1u << (TILE / EMB)) - 1u) {
