@@ -280,7 +280,9 @@ def _gpu_local_cpus(device_index):
 def bench_config(ev, name, args, peaks):
     """The step (probe + evidence over every layer) of one workload, timed on
     the launch stream with CUDA events: the whole step, and per layer the
-    probe call and the evidence call. Workloads whose inputs fit in L2 get a
+    probe call and the evidence call, once through each evidence path (the
+    text-row logit spill read back by the HBM-bound reduce, and the
+    recompute pass without the spill). Workloads whose inputs fit in L2 get a
     256 MB write before every timed step (outside the timed interval)."""
     import torch
     cfg = wl.CONFIGS[name]
@@ -308,49 +310,59 @@ def bench_config(ev, name, args, peaks):
     frames = total_vis // cfg.tokens_per_frame
     maps = [torch.zeros((hq, total_vis), device="cuda"), torch.zeros((hq, frames), device="cuda"),
             torch.zeros((len(probe.n_vis), hq), device="cuda"), torch.zeros((frames,), device="cuda")]
-    ws = ev.Workspace()
     stream = torch.cuda.current_stream()
-
-    def step(marks=None):
-        for layer, (q, k, v) in enumerate(dev):
-            if marks:
-                marks[layer][0].record(stream)
-            ev.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
-                                      probe.row_ptr, probe.col_idx, ws=ws, o=o, lse=lse)
-            if marks:
-                marks[layer][1].record(stream)
-            ev.evisel_evidence_reduce(ws, hq, probe.n_vis, cfg.tokens_per_frame, len(probe.n_vis), tok=maps[0],
-                                      frame=maps[1], head=maps[2], aqf=maps[3], accumulate=layer > 0)
-            if marks:
-                marks[layer][2].record(stream)
-
-    for _ in range(args.warmup):
-        step()
-    torch.cuda.synchronize()
-    if ev.evisel_status(ws) != 0:
-        raise RuntimeError(f"{name}: device status reported an error")
     ev_t = lambda: torch.cuda.Event(enable_timing=True)
-    bounds = [(ev_t(), ev_t()) for _ in range(args.steps)]
-    marks = [[[ev_t() for _ in range(3)] for _ in range(layers)] for _ in range(args.steps)]
-    for i in range(args.steps):
-        if flush_buf is not None:
-            flush_buf.zero_()
-        bounds[i][0].record(stream)
-        step(marks[i])
-        bounds[i][1].record(stream)
-    torch.cuda.synchronize()
-    status = ev.evisel_status(ws)
-    ws.free()
-    if status != 0:
-        raise RuntimeError(f"{name}: device status reported an error")
-    if not all(bool(torch.isfinite(m).all()) for m in maps):
-        raise RuntimeError(f"{name}: non-finite evidence maps")
-    step_ms = sum(a.elapsed_time(b) for a, b in bounds) / args.steps
-    attn_ms = sum(m[0].elapsed_time(m[1]) for s_ in marks for m in s_) / args.steps
-    ev_ms = sum(m[1].elapsed_time(m[2]) for s_ in marks for m in s_) / args.steps
+
+    def timed_steps(text_evidence):
+        """(step ms, probe ms, evidence ms) averaged over args.steps steps of one evidence path."""
+        ws = ev.Workspace()
+
+        def step(marks=None):
+            for layer, (q, k, v) in enumerate(dev):
+                if marks:
+                    marks[layer][0].record(stream)
+                ev.evisel_probe_attention(q, k, v, probe.cu_seqlens, probe.n_vis, cfg.tokens_per_frame, cfg.tile,
+                                          probe.row_ptr, probe.col_idx, ws=ws, o=o, lse=lse,
+                                          text_evidence=text_evidence)
+                if marks:
+                    marks[layer][1].record(stream)
+                ev.evisel_evidence_reduce(ws, hq, probe.n_vis, cfg.tokens_per_frame, len(probe.n_vis), tok=maps[0],
+                                          frame=maps[1], head=maps[2], aqf=maps[3], accumulate=layer > 0)
+                if marks:
+                    marks[layer][2].record(stream)
+
+        for _ in range(args.warmup):
+            step()
+        torch.cuda.synchronize()
+        if ev.evisel_status(ws) != 0:
+            raise RuntimeError(f"{name}: device status reported an error")
+        bounds = [(ev_t(), ev_t()) for _ in range(args.steps)]
+        marks = [[[ev_t() for _ in range(3)] for _ in range(layers)] for _ in range(args.steps)]
+        for i in range(args.steps):
+            if flush_buf is not None:
+                flush_buf.zero_()
+            bounds[i][0].record(stream)
+            step(marks[i])
+            bounds[i][1].record(stream)
+        torch.cuda.synchronize()
+        status = ev.evisel_status(ws)
+        ws_bytes = ws.nbytes
+        ws.free()
+        if status != 0:
+            raise RuntimeError(f"{name}: device status reported an error")
+        if not all(bool(torch.isfinite(m).all()) for m in maps):
+            raise RuntimeError(f"{name}: non-finite evidence maps")
+        step_ms = sum(a.elapsed_time(b) for a, b in bounds) / args.steps
+        attn_ms = sum(m[0].elapsed_time(m[1]) for s_ in marks for m in s_) / args.steps
+        ev_ms = sum(m[1].elapsed_time(m[2]) for s_ in marks for m in s_) / args.steps
+        return step_ms, attn_ms, ev_ms, ws_bytes
+
+    step_ms, attn_ms, ev_ms, _ = timed_steps(False)
+    rc_step_ms, rc_attn_ms, rc_ev_ms, rc_ws = timed_steps(True)
     flop = layers * st["flop"]
     attn_tflops = flop / (attn_ms * 1e-3) / 1e12
     ev_gbs = layers * st["evidence_bytes"] / (ev_ms * 1e-3) / 1e9
+    rc_attn_tflops = flop / (rc_attn_ms * 1e-3) / 1e12
     return {"workload": f"{cfg.name}: {cfg.description}", "tokens": st["n_tok"], "layers": layers,
             "videos": cfg.num_videos, "kept_tiles_per_layer": st["tiles"], "flop_per_step": flop,
             "step_ms": step_ms, "tflops": flop / (step_ms * 1e-3) / 1e12,
@@ -360,6 +372,14 @@ def bench_config(ev, name, args, peaks):
             "attention_ms_at_60pct_of_peak": flop / (0.6 * peaks["bf16"] * 1e12) * 1e3,
             "evidence_ms": ev_ms, "evidence_bytes": layers * st["evidence_bytes"], "evidence_gbs": ev_gbs,
             "evidence_frac_of_hbm": ev_gbs / peaks["hbm"],
+            "recompute_evidence": {
+                "note": "the same step with text_evidence = 1: the probe writes no text-row logit spill and the "
+                        "evidence call forms the text-row probabilities from q, k and the saved LSE",
+                "step_ms": rc_step_ms, "tflops": flop / (rc_step_ms * 1e-3) / 1e12,
+                "tokens_per_s": st["n_tok"] * layers / (rc_step_ms * 1e-3),
+                "attention_ms": rc_attn_ms, "attention_tflops": rc_attn_tflops,
+                "attention_frac_of_bf16_peak": rc_attn_tflops / peaks["bf16"],
+                "evidence_ms": rc_ev_ms, "workspace_bytes": rc_ws},
             "l2": "256 MB write before every step (untimed)" if flush else "inputs larger than L2 (no flush)"}
 
 
@@ -755,6 +775,14 @@ def bench_ours(args, cfg):
                           "attention_ms_at_60pct_of_peak": st["flop"] / (0.6 * peaks["bf16"] * 1e12) * 1e3,
                           "evidence_ms": ev_avg, "evidence_bytes": st["evidence_bytes"], "evidence_gbs": ev_gbs,
                           "evidence_frac_of_hbm": ev_gbs / peaks["hbm"], "l2": "inputs larger than L2 (no flush)",
+                          "recompute_evidence": {
+                              "note": "text_evidence_recompute above: the step without the text-row logit spill",
+                              "step_ms": te_step_ms, "tflops": st["flop"] / (te_step_ms * 1e-3) / 1e12,
+                              "tokens_per_s": st["n_tok"] / (te_step_ms * 1e-3),
+                              "attention_ms": te_probe_ms,
+                              "attention_tflops": st["flop"] / (te_probe_ms * 1e-3) / 1e12,
+                              "attention_frac_of_bf16_peak": st["flop"] / (te_probe_ms * 1e-3) / 1e12 / peaks["bf16"],
+                              "evidence_ms": te_ev_ms, "workspace_bytes": te_ws_bytes},
                           "note": "the headline step (value, attention, evidence above)"}
 
     line = None
@@ -797,7 +825,7 @@ def bench_ours(args, cfg):
                                          if local_cpus else "pinned (GPU NUMA node unknown)"),
                         "pipeline": "inputs of step i+1 and maps of step i copied on a second stream while "
                                     "step i computes"},
-                "gpu_launches": args.steps * (4 if _has_combine(probe) else 3),
+                "gpu_launches": args.steps * (4 if _has_combine(probe, torch.cuda.get_device_properties(local).multi_processor_count) else 3),
                 "clocks": clk,
                 "topp_sparse": topp_sparse,
                 "configs": configs}
@@ -816,15 +844,21 @@ def bench_ours(args, cfg):
     return 0
 
 
-def _has_combine(probe):
+def _has_combine(probe, sms):
+    """Whether the probe call launches the split-KV combine: some text row tile
+    has more kv tiles than the planner's split length (the longest visual row,
+    at least 8, raised to half of one SM's share of the tile work, capped at 64)."""
     cfg = probe.cfg
     counts = np.diff(probe.row_ptr)
-    split = max(int(counts.max()) if counts.size else 1, 8)
+    blocks = cfg.hkv * -(-(cfg.hq // cfg.hkv) // (2 * (128 // cfg.tile)))
+    work = int(counts.sum())
+    rows = []
     for nv, nt in zip(probe.n_vis, probe.n_text):
         n_vt, n_tt = -(-int(nv) // cfg.tile), -(-int(nt) // cfg.tile)
-        if n_tt and n_vt + n_tt > split:
-            return True
-    return False
+        rows += [n_vt + t + 1 for t in range(n_tt)]
+    work = (work + sum(rows)) * blocks
+    split = max(int(counts.max()) if counts.size else 1, 8, min(64, work // sms // 2))
+    return any(r > split for r in rows)
 
 
 def main():

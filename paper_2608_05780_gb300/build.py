@@ -29,7 +29,7 @@ LIB = os.path.join(HERE, "libevisel.so")
 SOURCES = ["probe_attn.cu", "attn_combine.cu", "evidence.cu", "evisel_capi.cpp", "evisel_noalloc.cu", "evisel_selftest.cu", "intra_frame.cu",
            "cross_frame.cu", "text_evidence.cu", "topp_mask.cu",
            "coarse_evidence.cu"]
-HEADERS = ["evisel_internal.h", "sm103_ptx.cuh"]
+HEADERS = ["evisel_internal.h", "evisel_plan.h", "sm103_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", "-I" + INCLUDE, "-I" + CSRC]

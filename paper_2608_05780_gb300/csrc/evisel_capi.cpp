@@ -15,6 +15,7 @@
 
 #include "../../include/evisel.h"
 #include "evisel_internal.h"
+#include "evisel_plan.h"
 
 using namespace evisel;
 
@@ -271,9 +272,15 @@ void build_plan(const evisel_probe_args* a, Plan& P) {
     P.aff_floats = off;
   }
 
-  // Text row tiles: dense causal over the video, split into chunks no longer
-  // than the longest visual row so that no CTA straggles.
-  const int split_len = std::max(max_visual, 8);
+  // Text row tiles: dense causal over the video, split into kv ranges of
+  // text_split_len tiles.
+  int64_t work = static_cast<int64_t>(P.kv.size());
+  for (int b = 0; b < a->num_videos; ++b) {
+    const VideoInfo& v = P.videos[b];
+    const int64_t n_vt = (v.n_vis + T - 1) / T, n_tt = (v.n_text + T - 1) / T;
+    work += n_tt * n_vt + n_tt * (n_tt + 1) / 2;
+  }
+  const int split_len = text_split_len(max_visual, work * static_cast<int64_t>(head_blocks.size()));
   for (int b = 0; b < a->num_videos; ++b) {
     const VideoInfo& v = P.videos[b];
     const int n_vt = (v.n_vis + T - 1) / T;

@@ -28,6 +28,7 @@
 
 #include "../../include/evisel.h"
 #include "evisel_internal.h"
+#include "evisel_plan.h"
 
 namespace evisel {
 int validate_probe_args(const evisel_probe_args* a);
@@ -67,8 +68,8 @@ struct Out {
 };
 
 // Work plan: one item per (query row tile, block of heads of one KV group, kv
-// range); text row tiles are split into kv ranges no longer than the longest
-// visual row. Counts only when `o` is null.
+// range); text row tiles are split into kv ranges of text_split_len tiles, as
+// in the allocating entry point. Counts only when `o` is null.
 void make_plan(const evisel_probe_args* a, Counts& c, const Out* o) {
   const int T = a->tile, hq = a->hq, gq = a->hq / a->hkv, hp = 128 / T;
   const int nb = a->num_videos;
@@ -117,7 +118,14 @@ void make_plan(const evisel_probe_args* a, Counts& c, const Out* o) {
                                               kv_begin, cnt, -1, b, -1};
     }
   }
-  const int split_len = std::max(max_visual, 8);
+  int64_t work = c.kv;
+  for (int b = 0; b < nb; ++b) {
+    const VideoInfo v = info(b);
+    const int64_t n_vt = (v.n_vis + T - 1) / T, n_tt = (v.n_text + T - 1) / T;
+    work += n_tt * n_vt + n_tt * (n_tt + 1) / 2;
+  }
+  const int64_t head_blocks = static_cast<int64_t>(a->hkv) * ((gq + kSlots * hp - 1) / (kSlots * hp));
+  const int split_len = text_split_len(max_visual, work * head_blocks);
   for (int b = 0; b < nb; ++b) {
     const VideoInfo v = info(b);
     const int n_vt = (v.n_vis + T - 1) / T;
