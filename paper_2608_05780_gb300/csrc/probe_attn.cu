@@ -11,7 +11,8 @@
 // Warp roles (352 threads):
 //   warps 0-3  softmax + epilogue of slot 0, one thread per query row (TMEM lane)
 //   warps 4-7  softmax + epilogue of slot 1
-//   warp 8     TMA: Q of both slots, then K_j into an NS-deep ring
+//   warp 8     block set-up (mbarriers) and the loads of Q (both slots) and
+//              K_0, before the block-wide barrier; then K_j into an NS-deep ring
 //   warp 10    TMA: V_j into an NS-deep ring (apart from K, so that K tiles
 //              run ahead of the V waits)
 //   warp 9     MMA issuer; the warp walks the tiles together and one elected
@@ -103,8 +104,51 @@ __device__ __forceinline__ int heads_left(const ProbeLaunch& L, int head) {
   return gq - head % gq;
 }
 
-// One TMA warp per ring, so that K tiles run ahead of the V waits: the K warp
-// also loads Q, the V warp only its ring.
+// Block set-up by the K loader's first lane, before the block-wide barrier:
+// the mbarriers and the abort flag, then the loads that the first S MMAs
+// wait for (Q of both slots and K tile 0), so that their latency overlaps the
+// TMEM allocation and the barrier instead of following them.
+template <int TILE, int D, int NS>
+__device__ __forceinline__ void setup_and_first_loads(const ProbeLaunch& L, const WorkItem& it, uint32_t sbase,
+                                                      volatile int* abort_flag) {
+  using C = Cfg<TILE, D, NS>;
+  auto bar = [&](int i) { return sbase + C::OFF_BAR + 8u * i; };
+  for (int i = 0; i < C::N_BARS; ++i) {
+    const bool softmax_arrive = (i == C::B_PF || i == C::B_PF + 1);
+    ptx::mbar_init(bar(i), softmax_arrive ? kRows : 1u);
+  }
+  *abort_flag = 0;
+  ptx::fence_mbar_init();
+  ptx::tma_prefetch_desc(&L.tm_q);
+  ptx::tma_prefetch_desc(&L.tm_k);
+  ptx::tma_prefetch_desc(&L.tm_v);
+  const int left = heads_left(L, it.head);
+  const int nslots = left > C::HP ? 2 : 1;
+  const uint64_t pol_q = ptx::l2_policy_evict_first();
+  ptx::mbar_arrive_expect_tx(bar(C::B_Q), nslots * C::Q_BYTES);
+  for (int slot = 0; slot < nslots; ++slot) {
+#pragma unroll
+    for (int hp = 0; hp < C::HP; ++hp) {
+      // A head past the group's end loads the first head again; its rows are never stored.
+      const int h = slot * C::HP + hp < left ? it.head + slot * C::HP + hp : it.head;
+#pragma unroll
+      for (int kb = 0; kb < C::KB; ++kb)
+        ptx::tma_load_3d(sbase + C::OFF_Q + slot * C::Q_BYTES + kb * C::Q_BLOCK + hp * TILE * 128, &L.tm_q,
+                         bar(C::B_Q), kb * 64, h, it.q_start, pol_q);
+    }
+  }
+  if (it.kv_count > 0) {
+    const int g = it.head / (L.hq / L.hkv);
+    ptx::mbar_arrive_expect_tx(bar(C::B_KF), C::KV_BYTES);
+#pragma unroll
+    for (int kb = 0; kb < C::KB; ++kb)
+      ptx::tma_load_3d(sbase + C::OFF_K + kb * C::KV_BLOCK, &L.tm_k, bar(C::B_KF), kb * 64, g,
+                       L.kv[it.kv_begin].start, ptx::l2_policy_evict_last());
+  }
+}
+
+// One TMA warp per ring, so that K tiles run ahead of the V waits. Q and K
+// tile 0 were sent by setup_and_first_loads; the K warp goes on from K tile 1.
 template <int TILE, int D, int NS, bool IS_V>
 __device__ __forceinline__ void producer(const ProbeLaunch& L, const WorkItem& it, uint32_t sbase_in,
                                          volatile int* abort_flag) {
@@ -112,40 +156,19 @@ __device__ __forceinline__ void producer(const ProbeLaunch& L, const WorkItem& i
   const uint32_t sbase = __shfl_sync(0xffffffffu, sbase_in, 0);
   auto bar = [&](int i) { return sbase + C::OFF_BAR + 8u * i; };
   const int head0 = __shfl_sync(0xffffffffu, it.head, 0);
-  const int q_start = __shfl_sync(0xffffffffu, it.q_start, 0);
   const int n = __shfl_sync(0xffffffffu, it.kv_count, 0);
   const int kv_begin = __shfl_sync(0xffffffffu, it.kv_begin, 0);
   const int g = head0 / (L.hq / L.hkv);
-  const int left = heads_left(L, head0);
-  const int nslots = left > C::HP ? 2 : 1;
-  const uint64_t pol_q = ptx::l2_policy_evict_first();
   const uint64_t pol_kv = ptx::l2_policy_evict_last();
   uint32_t leader = 0;
-  if (!IS_V && ptx::elect_one(leader)) {
-    ptx::tma_prefetch_desc(&L.tm_q);
-    ptx::tma_prefetch_desc(&L.tm_k);
-    ptx::tma_prefetch_desc(&L.tm_v);
-    ptx::mbar_arrive_expect_tx(bar(C::B_Q), nslots * C::Q_BYTES);
-    for (int slot = 0; slot < nslots; ++slot) {
-#pragma unroll
-      for (int hp = 0; hp < C::HP; ++hp) {
-        // A head past the group's end loads the first head again; its rows are never stored.
-        const int h = slot * C::HP + hp < left ? head0 + slot * C::HP + hp : head0;
-#pragma unroll
-        for (int kb = 0; kb < C::KB; ++kb)
-          ptx::tma_load_3d(sbase + C::OFF_Q + slot * C::Q_BYTES + kb * C::Q_BLOCK + hp * TILE * 128, &L.tm_q,
-                           bar(C::B_Q), kb * 64, h, q_start, pol_q);
-      }
-    }
-  }
-  __syncwarp();
 
   const CUtensorMap* map = IS_V ? &L.tm_v : &L.tm_k;
   const int off = IS_V ? C::OFF_V : C::OFF_K;
   const int b_full = IS_V ? C::B_VF : C::B_KF;
   const int b_empty = IS_V ? C::B_VE : C::B_KE;
-  int issued = 0;
-  for (int j = 0; j < n; ++j) {
+  const int first = (IS_V || n == 0) ? 0 : 1;   // K tile 0 went out with the set-up
+  int issued = first;
+  for (int j = first; j < n; ++j) {
     const int s = j % NS;
     const int u = j / NS;
     const int kv_start = __shfl_sync(0xffffffffu, L.kv[kv_begin + j].start, 0);
@@ -719,14 +742,7 @@ __global__ void __launch_bounds__(kThreads, 1) probe_attn_kernel(const __grid_co
   const int warp = threadIdx.x >> 5;
   const WorkItem it = L.items[blockIdx.x];
 
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < C::N_BARS; ++i) {
-      const bool softmax_arrive = (i == C::B_PF || i == C::B_PF + 1);
-      ptx::mbar_init(sbase + C::OFF_BAR + 8u * i, softmax_arrive ? kRows : 1u);
-    }
-    *abort_flag = 0;
-    ptx::fence_mbar_init();
-  }
+  if (threadIdx.x == kWarpProducer * 32) setup_and_first_loads<TILE, D, NS>(L, it, sbase, abort_flag);
   if (warp == 0) {
     ptx::tmem_alloc<C::TMEM_COLS>(ptx::smem_addr(tmem_slot));
     ptx::tmem_relinquish();
