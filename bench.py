@@ -159,9 +159,11 @@ class ClockSampler:
             return None
         sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
         smax = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        pw = [float(r[3]) for r in rows if r[3].strip().replace(".", "").isdigit()]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].strip() == "Active"})
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "sm_mhz_min": min(sm) if sm else None, "power_w_max": max(pw) if pw else None,
                 "reasons": reasons, "samples": len(rows)}
 
 
@@ -585,10 +587,13 @@ def bench_ours(args, cfg):
         dist.barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
+    e2e_clocks = ClockSampler(local)
+    e2e_clocks.start()
     e0.record(stream)
     e2e_run(args.steps, start_evt=e0)
     e1.record(stream)
     torch.cuda.synchronize()
+    e2e_clk = e2e_clocks.stop()
     e2e_ms = _max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     # the copies are done: the last step's maps are on the host
     if not all(np.isfinite(hm.numpy()).all() for hm in host_maps):
@@ -824,7 +829,8 @@ def bench_ours(args, cfg):
                         "host_buffers": (f"pinned, first touched on the GPU's {len(local_cpus)} local CPUs"
                                          if local_cpus else "pinned (GPU NUMA node unknown)"),
                         "pipeline": "inputs of step i+1 and maps of step i copied on a second stream while "
-                                    "step i computes"},
+                                    "step i computes",
+                        "clocks": e2e_clk},
                 "gpu_launches": args.steps * (4 if _has_combine(probe, torch.cuda.get_device_properties(local).multi_processor_count) else 3),
                 "clocks": clk,
                 "topp_sparse": topp_sparse,
