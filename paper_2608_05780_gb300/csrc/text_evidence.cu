@@ -10,7 +10,8 @@
 //   warp 4  TMA: the key tile K_g once, then Q_h of each text tile of the
 //           video for the group's heads, into a 2-deep ring (128B swizzle)
 //   warp 5  MMA: S^T = K_g Q_h^T (tcgen05, bf16 in, fp32 in TMEM; M = 128
-//           keys, N = 128 text rows) into a double-buffered TMEM tile
+//           keys, N = 128 text rows, 64 for a text tile of at most 64 rows)
+//           into a double-buffered TMEM tile
 //   warps 0-3  one thread per key (TMEM lane): adds exp2(s scale log2e -
 //           LSE log2e) over the 128 text-row columns of its lane (LSE of the
 //           step's text rows staged in shared memory), so no reduction
@@ -137,6 +138,9 @@ __global__ void __launch_bounds__(kThreads, 2) text_evidence_kernel(const __grid
       ptx::mbar_wait(bar(C::B_QF + s), ((issued - 1 - s) / C::QS) & 1, &never, kWaitTimeoutNs);
   } else if (warp == kWarpMma) {
     constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kRows, kRows, false, false);
+    // A text tile with at most 64 rows (the last, ragged tile of a video)
+    // takes an N = 64 MMA; the key threads read only those columns.
+    constexpr uint32_t kIdescHalf = ptx::idesc_bf16_f32(kRows, 64, false, false);
     uint32_t leader = 0;
     int first_leader = -1;
     bool same = true, issued = false, ok = true;
@@ -152,6 +156,7 @@ __global__ void __launch_bounds__(kThreads, 2) text_evidence_kernel(const __grid
       const bool me = ptx::elect_one(leader);
       if (first_leader < 0) first_leader = static_cast<int>(leader);
       same = same && static_cast<int>(leader) == first_leader;
+      const uint32_t idesc = vi.n_text - (t % n_tt) * kRows <= 64 ? kIdescHalf : kIdesc;
       if (me && same) {
         const uint32_t kbase = sbase + C::OFF_K;
         const uint32_t qbase = sbase + C::OFF_Q + (t % C::QS) * C::TILE_BYTES;
@@ -159,7 +164,7 @@ __global__ void __launch_bounds__(kThreads, 2) text_evidence_kernel(const __grid
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint64_t a = ptx::sdesc_sw128(kbase + (kk / 4) * C::BLOCK + (kk % 4) * 32, 16, 1024);
           const uint64_t bd = ptx::sdesc_sw128(qbase + (kk / 4) * C::BLOCK + (kk % 4) * 32, 16, 1024);
-          ptx::mma_ss(tmem + b * kRows, a, bd, kIdesc, kk > 0 ? 1u : 0u);
+          ptx::mma_ss(tmem + b * kRows, a, bd, idesc, kk > 0 ? 1u : 0u);
         }
         ptx::mma_commit(bar(C::B_SF + b));
         ptx::mma_commit(bar(C::B_QE + t % C::QS));
@@ -202,8 +207,10 @@ __global__ void __launch_bounds__(kThreads, 2) text_evidence_kernel(const __grid
         if (ok) {
           ptx::tc_fence_after();
           const float* lrow = lse_s + b * kRows;
+          const int valid = vi.n_text - tt * kRows;   // text rows in this tile; columns past them add 0
 #pragma unroll
           for (int c0 = 0; c0 < kRows; c0 += 64) {
+            if (c0 >= valid) break;                    // a 64-column half of padding rows only
             uint32_t r0[32], r1[32];
             ptx::tmem_ld32(tbase + b * kRows + c0, r0);
             ptx::tmem_ld32(tbase + b * kRows + c0 + 32, r1);
